@@ -1,0 +1,202 @@
+"""Reference oracle for the affinity-aware sharding hot path -- TEST INFRASTRUCTURE.
+
+A plain fp64 / exact-integer CPU statement of what the path computes, written
+from "Affinity-Aware Sharding for Delayed Tensor Parallelism" (arXiv
+2609.13846), Sec. 3 ("Affinity scores", "Objective", "Optimiser").  The C
+source is ``dtp_oracle.c``; this module compiles it with gcc and wraps it with
+ctypes and numpy.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline
+leg may import this package.  It shares no code with the CUDA library and
+imports nothing from it.
+
+Parity status: every function here is pinned by ``tests/test_oracle_*.py``
+(finite differences, closed forms, invariances, brute force, the Hungarian
+method, and the counts the paper prints).  Values the paper prints for its own
+models (the J values of Table 4) need the paper's weights and data and are
+unpinned.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "dtp_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lib = None
+
+_i64p = ctypes.POINTER(ctypes.c_int64)
+_i32p = ctypes.POINTER(ctypes.c_int)
+_f64p = ctypes.POINTER(ctypes.c_double)
+_f32p = ctypes.POINTER(ctypes.c_float)
+
+
+def build(force: bool = False) -> str:
+    """Compile ``dtp_oracle.c`` into ``liboracle.so`` (plain gcc, OpenMP)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", "-o", _LIB, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    lib = ctypes.CDLL(build())
+    lib.oracle_num_threads.restype = ctypes.c_int
+    lib.oracle_affinity_fo.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int,
+                                       ctypes.c_int, ctypes.c_int, _f64p]
+    lib.oracle_affinity_fo.restype = None
+    lib.oracle_finalize.argtypes = [_f64p, ctypes.c_int, ctypes.c_int, ctypes.c_int64, _f64p]
+    lib.oracle_finalize.restype = None
+    lib.oracle_quantize.argtypes = [_f32p, ctypes.c_int, ctypes.c_int, _i64p, _i32p]
+    lib.oracle_quantize.restype = ctypes.c_int
+    lib.oracle_layout_score.argtypes = [_i64p, ctypes.c_int, ctypes.c_int, _i32p, _i32p]
+    lib.oracle_layout_score.restype = ctypes.c_int64
+    lib.oracle_neuron_step_ex.argtypes = [_i64p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p,
+                                          _i32p, _i32p, ctypes.c_int]
+    lib.oracle_neuron_step_ex.restype = ctypes.c_int
+    lib.oracle_assignment_gain.argtypes = [_i64p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p]
+    lib.oracle_assignment_gain.restype = ctypes.c_int64
+    lib.oracle_count_partitions.argtypes = [ctypes.c_int, ctypes.c_int]
+    lib.oracle_count_partitions.restype = ctypes.c_int64
+    lib.oracle_head_step.argtypes = [_i64p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p, _i64p]
+    lib.oracle_head_step.restype = ctypes.c_int
+    lib.oracle_search_layout.argtypes = [_f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                         _i32p, _i32p, _i64p, _f64p, _i32p, _i32p]
+    lib.oracle_search_layout.restype = ctypes.c_int
+    lib.oracle_hungarian_max.argtypes = [_i64p, ctypes.c_int, _i32p]
+    lib.oracle_hungarian_max.restype = ctypes.c_int64
+    _lib = lib
+    return lib
+
+
+def _p(a: np.ndarray, ptype):
+    return a.ctypes.data_as(ptype)
+
+
+def _c(a, dtype) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=dtype))
+
+
+def num_threads() -> int:
+    """OpenMP threads the affinity oracle uses."""
+    return int(_load().oracle_num_threads())
+
+
+def affinity_fo(X, C, W_gate, W_up) -> np.ndarray:
+    """A[h,k] = sum_t Delta_{t,h,k}^2 in fp64 (Sec. 3, equation for Delta).
+
+    X [T,d], C [G,T,d], W_gate/W_up [N,d]; any real dtype, upcast exactly to fp64.
+    """
+    X = _c(X, np.float64)
+    C = _c(C, np.float64)
+    Wg = _c(W_gate, np.float64)
+    Wu = _c(W_up, np.float64)
+    T, d = X.shape
+    G = C.shape[0]
+    N = Wg.shape[0]
+    assert C.shape == (G, T, d) and Wg.shape == (N, d) and Wu.shape == (N, d)
+    A = np.zeros((G, N), dtype=np.float64)
+    _load().oracle_affinity_fo(_p(X, _f64p), _p(C, _f64p), _p(Wg, _f64p), _p(Wu, _f64p),
+                               T, d, G, N, _p(A, _f64p))
+    return A
+
+
+def finalize(A, T_total: int, wd_sqnorm=None) -> np.ndarray:
+    """A * ||w^d_k||^2 / T_total (Sec. 3: the E_t mean and the down-projection factor)."""
+    A = _c(A, np.float64).copy()
+    G, N = A.shape
+    wd = None if wd_sqnorm is None else _c(wd_sqnorm, np.float64)
+    _load().oracle_finalize(_p(A, _f64p), G, N, T_total, None if wd is None else _p(wd, _f64p))
+    return A
+
+
+def quantize(A):
+    """Exact fixed-point form of a layer's affinity: (q int64 [G,N], e)."""
+    A = _c(A, np.float32)
+    G, N = A.shape
+    q = np.zeros((G, N), dtype=np.int64)
+    e = ctypes.c_int(0)
+    st = _load().oracle_quantize(_p(A, _f32p), G, N, _p(q, _i64p), ctypes.byref(e))
+    if st != 0:
+        raise ValueError(f"oracle_quantize: status {st}")
+    return q, e.value
+
+
+def layout_score(q, h, nu) -> int:
+    """Integer up-edge co-located mass of a layout (Eq. objective, one layer)."""
+    q = _c(q, np.int64)
+    G, N = q.shape
+    return int(_load().oracle_layout_score(_p(q, _i64p), G, N, _p(_c(h, np.int32), _i32p),
+                                           _p(_c(nu, np.int32), _i32p)))
+
+
+def neuron_step(q, h, D: int, general: bool = False):
+    """Lexicographically smallest optimal balanced neuron assignment: (nu, unique)."""
+    q = _c(q, np.int64)
+    G, N = q.shape
+    nu = np.zeros(N, dtype=np.int32)
+    uniq = ctypes.c_int(0)
+    st = _load().oracle_neuron_step_ex(_p(q, _i64p), G, N, D, _p(_c(h, np.int32), _i32p),
+                                       _p(nu, _i32p), ctypes.byref(uniq), int(general))
+    if st != 0:
+        raise ValueError(f"oracle_neuron_step: status {st}")
+    return nu, bool(uniq.value)
+
+
+def assignment_gain(q, h, nu, D: int) -> int:
+    q = _c(q, np.int64)
+    G, N = q.shape
+    return int(_load().oracle_assignment_gain(_p(q, _i64p), G, N, D, _p(_c(h, np.int32), _i32p),
+                                              _p(_c(nu, np.int32), _i32p)))
+
+
+def count_partitions(G: int, D: int) -> int:
+    return int(_load().oracle_count_partitions(G, D))
+
+
+def head_step(q, nu, D: int):
+    """Best labelled balanced head partition given nu: (h, score)."""
+    q = _c(q, np.int64)
+    G, N = q.shape
+    h = np.zeros(G, dtype=np.int32)
+    s = ctypes.c_int64(0)
+    st = _load().oracle_head_step(_p(q, _i64p), G, N, D, _p(_c(nu, np.int32), _i32p), _p(h, _i32p),
+                                  ctypes.byref(s))
+    if st != 0:
+        raise ValueError(f"oracle_head_step: status {st}")
+    return h, int(s.value)
+
+
+def search_layout(A, D: int, iters: int):
+    """Coordinate ascent on one layer: dict(h, nu, score_q, score, iters_done, unique)."""
+    A = _c(A, np.float32)
+    G, N = A.shape
+    h = np.zeros(G, dtype=np.int32)
+    nu = np.zeros(N, dtype=np.int32)
+    sq = ctypes.c_int64(0)
+    sc = ctypes.c_double(0.0)
+    it = ctypes.c_int(0)
+    uq = ctypes.c_int(0)
+    st = _load().oracle_search_layout(_p(A, _f32p), G, N, D, iters, _p(h, _i32p), _p(nu, _i32p),
+                                      ctypes.byref(sq), ctypes.byref(sc), ctypes.byref(it),
+                                      ctypes.byref(uq))
+    if st != 0:
+        raise ValueError(f"oracle_search_layout: status {st}")
+    return dict(h=h, nu=nu, score_q=int(sq.value), score=float(sc.value), iters_done=int(it.value),
+                unique=bool(uq.value))
+
+
+def hungarian_max(W):
+    """Textbook Hungarian method: (max total, row_to_col) of a square int64 matrix."""
+    W = _c(W, np.int64)
+    n = W.shape[0]
+    r2c = np.zeros(n, dtype=np.int32)
+    total = _load().oracle_hungarian_max(_p(W, _i64p), n, _p(r2c, _i32p))
+    return int(total), r2c
