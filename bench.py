@@ -1,0 +1,337 @@
+"""Benchmark of the affinity-aware sharding hot path on GB300.
+
+One step = the whole hot path on one calibration layer of the Qwen3-0.6B
+shape (d=1024, 8 KV groups, SwiGLU N=3072, T=16384 tokens, D=2 devices):
+zero A, dtp_affinity_accumulate (tcgen05 bf16 GEMM with the fused SwiGLU
+first-order epilogue and on-chip token reduction), then dtp_search_layout
+(10 coordinate-ascent iterations).  Inputs (302 MB of activations) are larger
+than the 129 MB L2, so no flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank processes its own layer (seed + rank): the affinity
+pass and the up-edge search are independent per layer, so there is no
+collective on the data path ("weak" scaling); the timed region is bracketed by
+barriers and the max over ranks is reported.  ``--impl reference`` times the
+fp64 CPU oracle (the reference arm for this method) on a bounded token slice.
+Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_13846_gb300 import synth  # noqa: E402
+
+WORKLOAD = "qwen3_0.6b_layer"
+METRIC = "affinity tokens/s per layer (Qwen3-0.6B shape)"
+UNIT = "tokens/s"
+
+
+def flop_per_token(w) -> float:
+    """2*d*(2N)*(G+1): X and every C_h against [W_gate | W_up]."""
+    return 2.0 * w.d * 2 * w.N * (w.G + 1)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        j = json.load(open(p))
+        return dict(bf16=float(j["bf16_tflops"]), bf16_sustained=float(j.get("bf16_tflops_sustained", 0)),
+                    hbm=float(j["hbm_gbs"]), source="measured")
+    return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
+
+
+def traffic_from_profile():
+    """DRAM bytes per launch of the affinity kernel from the committed ncu summary, if current."""
+    p = os.path.join(ROOT, "profiles", "affinity_fo_tc_qwen3_layer.txt")
+    if not os.path.exists(p):
+        return None
+    for line in open(p):
+        if line.startswith("dram_bytes_per_full_launch:"):
+            try:
+                return float(line.split(":", 1)[1].split()[0])
+            except ValueError:
+                return None
+    return None
+
+
+class Clocks:
+    """Samples nvidia-smi clocks and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        os.unlink(self.path)
+        busy = [s for s in sm if smax and s > 0.3 * smax] or sm
+        return {"sm_mhz": statistics.median(busy) if busy else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_reference(args, w):
+    """The fp64 CPU oracle (the reference arm for this method) on a bounded token slice."""
+    import oracle
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    T_slice = args.cpu_tokens
+    L = synth.make_workload_layer(w, T=T_slice)
+    X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
+    for _ in range(args.warmup):
+        oracle.affinity_fo(X[:8], C[:, :8], Wg, Wu)
+    times = []
+    A = None
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        A = oracle.affinity_fo(X, C, Wg, Wu)
+        oracle.search_layout(A.astype(np.float32), w.D[0], w.iters)
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = T_slice * args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "d": w.d, "G": w.G, "N": w.N, "T": w.T, "D": w.D[0],
+                   "iters": w.iters, "token_slice": T_slice},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": f"{T_slice} of {w.T} tokens of one layer per step, then the D={w.D[0]} search"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def cpu_baseline(w, A_gpu, budget_s: float):
+    """Oracle timed on the host cores on a bounded token slice (rank 0, N=1 only)."""
+    import oracle
+    T0 = 16
+    L = synth.make_workload_layer(w, T=T0)
+    X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
+    t0 = time.perf_counter()
+    oracle.affinity_fo(X, C, Wg, Wu)
+    per_tok = (time.perf_counter() - t0) / T0
+    T_slice = int(max(T0, min(2048, budget_s / max(per_tok, 1e-9))))
+    L = synth.make_workload_layer(w, T=T_slice)
+    X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
+    t0 = time.perf_counter()
+    oracle.affinity_fo(X, C, Wg, Wu)
+    t_aff = time.perf_counter() - t0
+    A_np = A_gpu.float().cpu().numpy()
+    t0 = time.perf_counter()
+    oracle.search_layout(A_np, w.D[0], w.iters)
+    t_search = time.perf_counter() - t0
+    return {"value": T_slice / t_aff, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"affinity on {T_slice} of {w.T} tokens of one layer (fp64); "
+                      f"search on the GPU's A took {1e3 * t_search:.1f} ms",
+            "search_ms": 1e3 * t_search}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--cpu-tokens", type=int, default=64, help="token slice per step of --impl reference")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    w = synth.WORKLOADS[WORKLOAD]
+
+    if args.impl == "reference":
+        run_reference(args, w)
+        return
+
+    from paper_2609_13846_gb300 import dtp
+
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    peaks = load_peaks()
+
+    # inputs resident in HBM; each rank owns one layer
+    L = synth.make_layer(w.d, w.G, w.N, w.T, w.seed + rank, dtype=w.dtype, outliers=w.outliers, device=dev)
+    X, C, Wg, Wu = L["X"], L["C"], L["W_gate"], L["W_up"]
+    D, iters = w.D[0], w.iters
+    A = torch.zeros((w.G, w.N), dtype=torch.float32, device=dev)
+    ws_aff = dtp.affinity_workspace(w.T, w.d, w.G, w.N, dtp.DTP_BF16, dev)
+    ws_search = torch.empty(dtp.search_workspace_size(1, w.G, w.N, D), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    aff_ev = []
+
+    def step(record=False):
+        A.zero_()
+        if record:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        dtp.affinity_accumulate(X, C, Wg, Wu, A=A, workspace=ws_aff)
+        if record:
+            e1.record(stream)
+            aff_ev.append((e0, e1))
+        return dtp.search_layout(A, D, iters, workspace=ws_search)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    if dtp.workspace_status(ws_aff) != dtp.DTP_OK:
+        raise RuntimeError("affinity kernel reported a wait timeout")
+
+    # ---- timed region: inputs resident on the device
+    barrier()
+    torch.cuda.synchronize()
+    with Clocks(local) as clk:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(args.steps):
+            res = step(record=True)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    elapsed_ms = t0.elapsed_time(t1)
+    aff_ms = [a.elapsed_time(b) for a, b in aff_ev]
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    ms_step = elapsed_ms / args.steps
+    value = world * w.T * args.steps / (elapsed_ms / 1e3)
+    clocks = clk.summary()
+
+    # search alone (same A, same launch) for the "search ms" part of the metric
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    for _ in range(5):
+        dtp.search_layout(A, D, iters, workspace=ws_search)
+    s1.record(stream)
+    torch.cuda.synchronize()
+    search_ms = s0.elapsed_time(s1) / 5
+
+    # ---- end to end through the public API, host buffers in pinned memory
+    hostL = {k: v.cpu().pin_memory() for k, v in L.items()}
+    h2d = sum(v.numel() * v.element_size() for v in hostL.values())
+    e2e_steps = max(3, min(args.steps, 10))
+    barrier()
+    torch.cuda.synchronize()
+    w0 = time.perf_counter()
+    d2h = 0
+    for _ in range(e2e_steps):
+        dX = hostL["X"].to(dev, non_blocking=True)
+        dC = hostL["C"].to(dev, non_blocking=True)
+        dWg = hostL["W_gate"].to(dev, non_blocking=True)
+        dWu = hostL["W_up"].to(dev, non_blocking=True)
+        Ae = dtp.affinity_accumulate(dX, dC, dWg, dWu, workspace=ws_aff)
+        r = dtp.search_layout(Ae, D, iters, workspace=ws_search)
+        outs = [Ae.cpu(), r["h"].cpu(), r["nu"].cpu(), r["score"].cpu()]
+        d2h = sum(o.numel() * o.element_size() for o in outs)
+    torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - w0
+    barrier()
+    e2e_value = world * w.T * e2e_steps / e2e_s
+
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    if rank != 0:
+        return
+
+    aff_mean_ms = float(np.mean(aff_ms))
+    fl = flop_per_token(w) * w.T
+    achieved = fl / (aff_mean_ms / 1e3) / 1e12
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"], "unit": "TFLOP/s",
+                "frac": achieved / peaks["bf16"], "traffic": traffic_from_profile(),
+                "kernel": "affinity_fo_tc_kernel (+ its partial-sum reduce)",
+                "peak_source": f"{peaks['source']} bf16 burst (cuBLAS 8192^3)",
+                "frac_of_sustained": achieved / peaks["bf16_sustained"] if peaks["bf16_sustained"] else None}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "d": w.d, "G": w.G, "N": w.N, "T": w.T, "D": D, "iters": iters,
+                   "layers_per_step": world, "l2": "inputs (302 MB) larger than L2; no flush"},
+        "affinity_ms": aff_mean_ms, "affinity_tflops": achieved, "search_ms": search_ms,
+        "search_iters_done": int(res["iters_done"]), "layout_score": float(res["score"]),
+        "roofline": roofline,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, A, args.cpu_budget)
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,179 @@
+/*
+ * dtp.h -- C ABI of libdtp, the GB300 (sm_103a) hot path of affinity-aware
+ * sharding for Delayed Tensor Parallelism ("Affinity-Aware Sharding for
+ * Delayed Tensor Parallelism", arXiv 2609.13846).
+ *
+ * Two parts, both defined in Sec. 3 of the paper:
+ *   1. the first-order head->neuron affinity of one layer ("Affinity scores"),
+ *   2. the coordinate-ascent layout optimiser over balanced head partitions
+ *      and neuron assignments ("Objective", "Optimiser").
+ *
+ * Conventions for every entry point:
+ *   - Tensor arguments are DEVICE pointers owned by the caller; the library
+ *     never frees or retains them.  Scratch memory is passed in as a
+ *     caller-owned device workspace whose size the *_workspace_size query
+ *     returns.  The library allocates no device memory.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Calls are asynchronous on it unless stated otherwise.
+ *   - Arrays are row-major, contiguous, 16-byte aligned.
+ *   - Every call returns a dtp_status; no C++ exception crosses the ABI.
+ *     Argument errors are found on the host before anything is launched and
+ *     leave every output untouched.
+ *   - Calls on different streams with disjoint outputs and workspaces may run
+ *     concurrently; a workspace must not be shared by calls in flight.
+ */
+#ifndef DTP_H_
+#define DTP_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DTP_OK = 0,
+    DTP_ERR_ARG = -1,            /* invalid size, pointer, alignment or combination      */
+    DTP_ERR_CUDA = -2,           /* a CUDA runtime/driver call failed                      */
+    DTP_ERR_NOT_CONVERGED = -3,  /* a bounded device loop or wait hit its limit            */
+    DTP_ERR_UNSUPPORTED = -4,    /* valid request this build does not handle (e.g. no GPU) */
+    DTP_ERR_WORKSPACE = -5       /* workspace NULL or smaller than the size query's value  */
+} dtp_status;
+
+typedef enum {
+    DTP_BF16 = 0, /* bf16 operands, fp32 accumulation (tcgen05 tensor cores)      */
+    DTP_F32 = 1   /* fp32 operands and arithmetic (CUDA cores; tight-check mode) */
+} dtp_dtype;
+
+/* Library version as major*10000 + minor*100 + patch. */
+int dtp_version(void);
+
+/* Static, human-readable text for a dtp_status value. */
+const char* dtp_status_string(int status);
+
+/* ------------------------------------------------------------------------ */
+/* 1. First-order affinity (Sec. 3 "Affinity scores")                        */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Bytes of device workspace dtp_affinity_accumulate needs for these sizes and
+ * dtype (written to *bytes).  Returns DTP_ERR_ARG for invalid sizes.
+ */
+int dtp_affinity_workspace_size(int64_t T, int d, int H_kv, int N, int dtype, size_t* bytes);
+
+/*
+ * A[h,k] += sum_{t<T} Delta_{t,h,k}^2, the first-order damage to SwiGLU
+ * neuron k's output silu(g_k) u_k from removing KV head h's piece of the FFN
+ * input (Sec. 3, the equation for Delta_hk):
+ *     g = x_t . w^g_k,  u = x_t . w^u_k,  pg = c_{h,t} . w^g_k,  pu = c_{h,t} . w^u_k
+ *     Delta = silu'(g) u pg + silu(g) pu,   silu'(g) = s (1 + g (1 - s)),  s = 1/(1+e^-g)
+ *
+ *   X       [T, d]        FFN input after the pre-norm (x / r * gamma), dtype
+ *   C       [H_kv, T, d]  each KV group's piece p_h of that input, in the same
+ *                         (post-norm) units, dtype
+ *   W_gate  [N, d]        gate projection rows w^g_k (nn.Linear [out, in]), dtype
+ *   W_up    [N, d]        up projection rows w^u_k, dtype
+ *   A       [H_kv, N]     fp32, ACCUMULATED (zero it before the first chunk);
+ *                         token chunks of one layer can therefore be streamed
+ *                         through successive calls
+ *   workspace             device scratch of at least
+ *                         dtp_affinity_workspace_size(...) bytes
+ *
+ * The E_t mean and the ||w^d_k||^2 factor of the paper's S^{up,fo} are applied
+ * by dtp_affinity_finalize.  The result is deterministic: the same inputs give
+ * bitwise the same A (no floating-point atomics).
+ * Requirements: T >= 0 (T == 0 returns DTP_OK at once and accepts NULL
+ * pointers), d >= 8 and d % 8 == 0 (16-byte rows), 1 <= H_kv <= 16, N >= 1,
+ * all pointers 16-byte aligned.
+ * Asynchronous on `stream`.  A device-side wait that exceeds its limit sets
+ * the workspace status word (see dtp_workspace_status).
+ */
+int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, const void* W_up,
+                            int64_t T, int d, int H_kv, int N, int dtype, float* A,
+                            void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * A[h,k] *= wd_sqnorm[k] / T_total, the token mean E_t and the squared norm of
+ * neuron k's down-projection column (Sec. 3, S^{up,fo} = E_t[Delta^2] ||w^d_k||^2).
+ * wd_sqnorm: device fp32 [N], or NULL for a factor of 1.  T_total >= 1.
+ * Both factors are positive, so neither changes the layout the optimiser finds
+ * except through the per-neuron ||w^d_k||^2.  Asynchronous on `stream`.
+ */
+int dtp_affinity_finalize(float* A, int H_kv, int N, int64_t T_total, const float* wd_sqnorm,
+                          void* stream);
+
+/*
+ * out[k] = sum_i W_down[i,k]^2 = ||w^d_k||^2 for W_down [d, N] (nn.Linear
+ * [out=d, in=N]) of the given dtype; out is device fp32 [N].  The input of
+ * dtp_affinity_finalize (Sec. 3, "w^d_k the down-projection column").
+ */
+int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, void* stream);
+
+/*
+ * Synchronises `stream`, then reads the status word that kernels of the last
+ * call using `workspace` leave in it: DTP_OK, or DTP_ERR_NOT_CONVERGED if a
+ * bounded device-side wait gave up.  workspace_bytes as passed to that call.
+ */
+int dtp_workspace_status(const void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* 2. Layout optimiser (Sec. 3 "Objective", "Optimiser")                     */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Bytes of device workspace dtp_search_layout(_batched) needs for `layers`
+ * layers of [H_kv, N] affinities over D devices.
+ */
+int dtp_search_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes);
+
+/*
+ * Coordinate ascent on the up-edge objective of one layer (Sec. 3):
+ *   J(h, nu) = sum over (g,k) with h(g) == nu(k) of S[g,k] / sum S,
+ * over balanced layouts: h assigns H_kv/D KV groups and nu assigns N/D neurons
+ * to each of the D devices.
+ *
+ *   - Exact arithmetic: the layer's matrix is mapped to the fixed-point form
+ *     q[g,k] = floor(A[g,k] * 2^(40-e)), max(A) < 2^e; unit-mass normalisation
+ *     is a positive scale and is applied only to the reported score.
+ *   - Start: contiguous heads h(g) = floor(g*D/H_kv).
+ *   - Iteration: neuron step (the optimal balanced assignment nu given h; the
+ *     gain of neuron k on device l is M[k,l] = sum over g with h(g) == l of
+ *     q[g,k]), then head step (the best of all H_kv!/((H_kv/D)!)^D labelled
+ *     balanced partitions given nu).
+ *   - Ties: the lexicographically smallest optimal nu, and the
+ *     lexicographically smallest best h.
+ *   - Stop after `iters` iterations or after the first iteration whose
+ *     integer score does not strictly exceed the previous one.
+ *
+ *   A           [H_kv, N] fp32, device, finite and >= 0
+ *   head_part   [H_kv] int32 out (device): h(g) in 0..D-1
+ *   neuron_dev  [N] int32 out (device): nu(k) in 0..D-1
+ *   score_q     int64 out (device): co-located fixed-point mass
+ *   score       double out (device): score_q / sum(q), in [0,1] (0 if A == 0)
+ *   iters_done  int32 out (device): iterations run (1..iters)
+ * Requirements: 2 <= D <= 8, D | H_kv, D | N, H_kv <= 16, N <= 262144,
+ * H_kv * N <= 4194304, iters >= 1, the partition count <= 2^26.
+ * SYNCHRONOUS: returns after the result is on the device and its status has
+ * been read; DTP_ERR_ARG also reports a negative or non-finite entry of A.
+ */
+int dtp_search_layout(const float* A, int H_kv, int N, int D, int iters,
+                      int32_t* head_part, int32_t* neuron_dev, int64_t* score_q, double* score,
+                      int32_t* iters_done, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * dtp_search_layout on `layers` independent layers at once (the up-edge
+ * objective decouples across layers); layer i reads A + i*H_kv*N and writes
+ * head_part + i*H_kv, neuron_dev + i*N, score_q[i], score[i], iters_done[i].
+ * One thread block per layer.  SYNCHRONOUS; returns the first failing
+ * layer's status.
+ */
+int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D, int iters,
+                              int32_t* head_part, int32_t* neuron_dev, int64_t* score_q,
+                              double* score, int32_t* iters_done, void* workspace,
+                              size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DTP_H_ */

@@ -1,0 +1,140 @@
+// dtp_api.cu -- the extern "C" entry points declared in include/dtp.h:
+// argument validation on the host, then dispatch to the kernels.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dtp_common.cuh"
+
+namespace dtp {
+namespace tc {
+size_t workspace_bytes(int64_t T, int d, int G, int N);
+int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
+           void* workspace, cudaStream_t stream);
+}  // namespace tc
+namespace f32 {
+size_t workspace_bytes(int64_t T, int d, int G, int N);
+int launch(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
+           float* A, void* workspace, cudaStream_t stream);
+}  // namespace f32
+int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream);
+int launch_down_sqnorm(const void* W, int d, int N, int dtype, float* out, cudaStream_t stream);
+namespace search {
+size_t workspace_bytes(int layers, int G, int N, int D);
+int64_t partition_count(int G, int D);
+int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* head, int32_t* nu, int64_t* score_q,
+           double* score, int32_t* iters_done, void* workspace, cudaStream_t stream);
+}  // namespace search
+}  // namespace dtp
+
+using namespace dtp;
+
+namespace {
+
+constexpr int kMaxHeads = 16;
+
+bool affinity_sizes_ok(int64_t T, int d, int H, int N, int dtype) {
+    if (dtype != DTP_BF16 && dtype != DTP_F32) return false;
+    if (T < 0 || d < 8 || (d % 8) != 0 || H < 1 || H > kMaxHeads || N < 1) return false;
+    // TMA coordinates are int32 and the token axis of C is addressed in one box dimension
+    if (T > (int64_t(1) << 31) - 256 || N > (1 << 30)) return false;
+    return true;
+}
+
+size_t affinity_ws(int64_t T, int d, int H, int N, int dtype) {
+    return dtype == DTP_BF16 ? tc::workspace_bytes(T, d, H, N) : f32::workspace_bytes(T, d, H, N);
+}
+
+bool search_sizes_ok(int layers, int H, int N, int D, int iters) {
+    if (layers < 1 || D < 2 || D > 8 || H < 1 || H > kMaxHeads || N < 1 || iters < 1) return false;
+    if (H % D || N % D) return false;
+    if (N > (1 << 18) || static_cast<int64_t>(H) * N > (int64_t(1) << 22)) return false;
+    if (search::partition_count(H, D) > (int64_t(1) << 26)) return false;
+    return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dtp_version(void) { return 100; }
+
+const char* dtp_status_string(int status) {
+    switch (status) {
+        case DTP_OK: return "ok";
+        case DTP_ERR_ARG: return "invalid argument";
+        case DTP_ERR_CUDA: return "CUDA error";
+        case DTP_ERR_NOT_CONVERGED: return "bounded device loop or wait hit its limit";
+        case DTP_ERR_UNSUPPORTED: return "unsupported";
+        case DTP_ERR_WORKSPACE: return "workspace missing or too small";
+        default: return "unknown status";
+    }
+}
+
+int dtp_affinity_workspace_size(int64_t T, int d, int H_kv, int N, int dtype, size_t* bytes) {
+    if (!bytes || !affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
+    *bytes = affinity_ws(T, d, H_kv, N, dtype);
+    return DTP_OK;
+}
+
+int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, const void* W_up, int64_t T, int d,
+                            int H_kv, int N, int dtype, float* A, void* workspace, size_t workspace_bytes,
+                            void* stream) {
+    if (!affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;  // nothing to add; empty inputs may have null data pointers
+    if (!X || !C || !W_gate || !W_up || !A) return DTP_ERR_ARG;
+    if (!aligned16(X) || !aligned16(C) || !aligned16(W_gate) || !aligned16(W_up) || !aligned16(A))
+        return DTP_ERR_ARG;
+    const size_t need = affinity_ws(T, d, H_kv, N, dtype);
+    if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    if (dtype == DTP_BF16) return tc::launch(X, C, W_gate, W_up, T, d, H_kv, N, A, workspace, s);
+    return f32::launch(static_cast<const float*>(X), static_cast<const float*>(C), static_cast<const float*>(W_gate),
+                       static_cast<const float*>(W_up), T, d, H_kv, N, A, workspace, s);
+}
+
+int dtp_affinity_finalize(float* A, int H_kv, int N, int64_t T_total, const float* wd_sqnorm, void* stream) {
+    if (!A || H_kv < 1 || H_kv > kMaxHeads || N < 1 || T_total < 1 || !aligned16(A)) return DTP_ERR_ARG;
+    return launch_finalize(A, H_kv, N, T_total, wd_sqnorm, static_cast<cudaStream_t>(stream));
+}
+
+int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, void* stream) {
+    if (!W_down || !out || d < 1 || N < 1 || (dtype != DTP_BF16 && dtype != DTP_F32)) return DTP_ERR_ARG;
+    return launch_down_sqnorm(W_down, d, N, dtype, out, static_cast<cudaStream_t>(stream));
+}
+
+int dtp_workspace_status(const void* workspace, size_t workspace_bytes, void* stream) {
+    if (!workspace || workspace_bytes < kWorkspaceHeader) return DTP_ERR_WORKSPACE;
+    int st = 0;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemcpyAsync(&st, workspace, sizeof(int), cudaMemcpyDeviceToHost, s));
+    DTP_CUDA_TRY(cudaStreamSynchronize(s));
+    return st == 0 ? DTP_OK : st;
+}
+
+int dtp_search_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes) {
+    if (!bytes || !search_sizes_ok(layers, H_kv, N, D, 1)) return DTP_ERR_ARG;
+    *bytes = search::workspace_bytes(layers, H_kv, N, D);
+    return DTP_OK;
+}
+
+int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D, int iters, int32_t* head_part,
+                              int32_t* neuron_dev, int64_t* score_q, double* score, int32_t* iters_done,
+                              void* workspace, size_t workspace_bytes, void* stream) {
+    if (!search_sizes_ok(layers, H_kv, N, D, iters)) return DTP_ERR_ARG;
+    if (!A || !head_part || !neuron_dev || !score_q || !score || !iters_done) return DTP_ERR_ARG;
+    if (!aligned16(A)) return DTP_ERR_ARG;
+    const size_t need = search::workspace_bytes(layers, H_kv, N, D);
+    if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    return search::launch(A, layers, H_kv, N, D, iters, head_part, neuron_dev, score_q, score, iters_done, workspace,
+                          static_cast<cudaStream_t>(stream));
+}
+
+int dtp_search_layout(const float* A, int H_kv, int N, int D, int iters, int32_t* head_part, int32_t* neuron_dev,
+                      int64_t* score_q, double* score, int32_t* iters_done, void* workspace, size_t workspace_bytes,
+                      void* stream) {
+    return dtp_search_layout_batched(A, 1, H_kv, N, D, iters, head_part, neuron_dev, score_q, score, iters_done,
+                                     workspace, workspace_bytes, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,658 @@
+// search.cu -- the layout optimiser of Sec. 3 ("Objective", "Optimiser") on
+// the GPU: coordinate ascent over balanced head partitions h and balanced
+// neuron assignments nu of one layer, maximising the co-located up-edge mass.
+//
+// One thread block (1024 threads) per layer; the layers of a batch are
+// independent because the up-edge objective decouples across layers.
+//
+// Exactness.  A is mapped to q[g,k] = floor(A[g,k] * 2^(40-e)) (max A < 2^e),
+// computed from the fp32 bit pattern with integer shifts, and every score is
+// an int64 sum, so no summation order can change a decision.
+//
+// Neuron step (exact balanced linear assignment, lexicographically smallest
+// optimum), gain M[k,l] = sum over heads g with h(g) == l of q[g,k]:
+//   D == 2  device 0 takes the N/2 largest M[k,0]-M[k,1], lower index first on
+//           ties: one block-wide radix selection of packed (difference, index)
+//           keys.
+//   D >  2  (a) device prices pi from a few Gauss-Seidel sweeps, each price set
+//           by a radix selection so that about N/D neurons prefer its device;
+//           (b) every neuron to its best device at those prices -- optimal for
+//           the resulting device counts by complementary slackness;
+//           (c) successive shortest paths on the D-node exchange graph
+//           (w[a][b] = best gain of moving one neuron from a to b) move one
+//           unit of excess per path until all counts equal N/D: each path is
+//           a maximum-gain path, so optimality for the counts is kept and the
+//           final assignment is optimal;
+//           (d) canonicalisation: for k = 0, 1, ..., move k to the smallest
+//           device l < nu(k) that a zero-gain exchange cycle through neurons
+//           > k allows; the result is the lexicographically smallest optimum.
+// Head step: B[g,l] = sum over neurons on l of q[g,k]; every labelled balanced
+// partition (H!/((H/D)!)^D of them) is scored by a slice of the block and the
+// best, lexicographically smallest on ties, is kept.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dtp_common.cuh"
+
+namespace dtp {
+namespace search {
+
+constexpr int kThreads = 1024;
+constexpr int kWarps = kThreads / 32;
+constexpr int DMAX = 8;
+constexpr int GMAX = 16;
+constexpr int kFixedBits = 40;
+constexpr int kIdxBits = 18;                       // N <= 2^18
+constexpr int64_t kValBias = int64_t(1) << 45;     // |gain| < 2^44 (H_kv <= 16): fits the 46-bit field
+constexpr int64_t kNegInf = INT64_MIN / 4;
+constexpr size_t kSmemBudget = 200 * 1024;         // dynamic smem for M and nu
+
+struct Shared {
+    uint64_t w[DMAX][DMAX];        // exchange-graph keys (0 = no neuron on the source device)
+    int64_t P[DMAX][DMAX];         // all-pairs max-gain paths
+    int64_t B[GMAX * DMAX];        // head-step column sums
+    int64_t pi[DMAX];              // device prices
+    int count[DMAX];
+    unsigned int hist[256];
+    int64_t red_i64[kWarps];
+    int red_int[kWarps];
+    uint64_t sel_prefix;
+    long long sel_rank;
+    int64_t total, J, Jprev;
+    int h[GMAX];
+    int status;
+    int flag;
+    int kstar;
+    int best_idx;
+};
+
+// ---------------------------------------------------------------- helpers --
+
+// floor(a * 2^(40-e)) for a finite a >= 0, by shifting the fp32 significand.
+__device__ __forceinline__ int64_t quantize(float a, int e) {
+    const uint32_t b = __float_as_uint(a);
+    const uint32_t ex = (b >> 23) & 0xFFu;
+    uint64_t m = b & 0x7FFFFFu;
+    int E;
+    if (ex == 0) {
+        E = -149;
+    } else {
+        m |= 0x800000u;
+        E = static_cast<int>(ex) - 150;
+    }
+    const int s = E + kFixedBits - e;
+    if (s >= 0) return static_cast<int64_t>(m << s);
+    if (s <= -40) return 0;
+    return static_cast<int64_t>(m >> (-s));
+}
+
+__device__ __forceinline__ uint64_t pack_gain(int64_t v, int k) {
+    return (static_cast<uint64_t>(v + kValBias) << kIdxBits) |
+           static_cast<uint64_t>((1 << kIdxBits) - 1 - k);
+}
+__device__ __forceinline__ int64_t gain_of(uint64_t key) {
+    return static_cast<int64_t>(key >> kIdxBits) - kValBias;
+}
+__device__ __forceinline__ int index_of(uint64_t key) {
+    return (1 << kIdxBits) - 1 - static_cast<int>(key & ((1u << kIdxBits) - 1));
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t x) {
+    const uint32_t hi = static_cast<uint32_t>(x >> 32);
+    const uint32_t mhi = __reduce_max_sync(0xFFFFFFFFu, hi);
+    const uint32_t lo = (hi == mhi) ? static_cast<uint32_t>(x) : 0u;
+    const uint32_t mlo = __reduce_max_sync(0xFFFFFFFFu, lo);
+    return (static_cast<uint64_t>(mhi) << 32) | mlo;
+}
+
+__device__ __forceinline__ int64_t warp_sum_i64(int64_t x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    return x;
+}
+
+__device__ int64_t block_sum_i64(int64_t x, Shared& sh) {
+    x = warp_sum_i64(x);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) sh.red_i64[warp] = x;
+    __syncthreads();
+    int64_t t = 0;
+    for (int i = 0; i < kWarps; ++i) t += sh.red_i64[i];
+    return t;
+}
+
+__device__ int64_t block_max_i64(int64_t x, Shared& sh) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const int64_t y = __shfl_xor_sync(0xFFFFFFFFu, x, o);
+        x = y > x ? y : x;
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) sh.red_i64[warp] = x;
+    __syncthreads();
+    int64_t t = sh.red_i64[0];
+    for (int i = 1; i < kWarps; ++i) t = sh.red_i64[i] > t ? sh.red_i64[i] : t;
+    return t;
+}
+
+__device__ int block_min_int(int x, Shared& sh) {
+    x = static_cast<int>(__reduce_min_sync(0xFFFFFFFFu, static_cast<unsigned>(x)));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) sh.red_int[warp] = x;
+    __syncthreads();
+    int t = sh.red_int[0];
+    for (int i = 1; i < kWarps; ++i) t = sh.red_int[i] < t ? sh.red_int[i] : t;
+    return t;
+}
+
+// The r-th largest (1-based) of the n keys key(0..n-1), by an 8-bit
+// most-significant-digit radix selection.  Collective over the block.
+template <class KeyFn>
+__device__ uint64_t block_select_desc(int n, long long r, KeyFn key, Shared& sh) {
+    uint64_t prefix = 0;
+    if (threadIdx.x == 0) sh.sel_rank = r;
+    for (int shift = 56; shift >= 0; shift -= 8) {
+        for (int i = threadIdx.x; i < 256; i += kThreads) sh.hist[i] = 0;
+        __syncthreads();
+        const uint64_t hi_mask = (shift == 56) ? 0ull : (~0ull << (shift + 8));
+        for (int i = threadIdx.x; i < n; i += kThreads) {
+            const uint64_t kv = key(i);
+            const bool match = (kv & hi_mask) == (prefix & hi_mask);
+            const unsigned bin = match ? static_cast<unsigned>((kv >> shift) & 255u) : 256u;
+            const unsigned peers = __match_any_sync(__activemask(), bin);
+            if (match && (__ffs(peers) - 1) == (threadIdx.x & 31)) atomicAdd(&sh.hist[bin], __popc(peers));
+        }
+        __syncthreads();
+        if (threadIdx.x < 32) {
+            // lane L owns bins [248 - 8L, 255 - 8L], scanned from the top
+            const int lane = threadIdx.x;
+            unsigned cnt = 0;
+            for (int b = 0; b < 8; ++b) cnt += sh.hist[255 - 8 * lane - b];
+            unsigned incl = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const unsigned y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const long long rr = sh.sel_rank;
+            const bool here = (incl >= rr) && (incl - cnt < rr);
+            const unsigned who = __ballot_sync(0xFFFFFFFFu, here);
+            if (here) {
+                long long left = rr - static_cast<long long>(incl - cnt);
+                for (int b = 0; b < 8; ++b) {
+                    const int bin = 255 - 8 * lane - b;
+                    if (left <= static_cast<long long>(sh.hist[bin])) {
+                        sh.sel_prefix = prefix | (static_cast<uint64_t>(bin) << shift);
+                        sh.sel_rank = left;
+                        break;
+                    }
+                    left -= sh.hist[bin];
+                }
+            }
+            if (who == 0u && lane == 0) sh.status = DTP_ERR_NOT_CONVERGED;  // rank out of range
+        }
+        __syncthreads();
+        prefix = sh.sel_prefix;
+        __syncthreads();
+    }
+    return prefix;
+}
+
+struct Layer {
+    const float* A;
+    int G, N, D, cap, e;
+    int64_t* M;   // [N][D]
+    int32_t* nu;  // [N]
+};
+
+__device__ void build_gain(const Layer& L, Shared& sh) {
+    for (int k = threadIdx.x; k < L.N; k += kThreads) {
+        int64_t m[DMAX];
+#pragma unroll
+        for (int l = 0; l < DMAX; ++l) m[l] = 0;
+        for (int g = 0; g < L.G; ++g) {
+            const int64_t q = quantize(L.A[static_cast<int64_t>(g) * L.N + k], L.e);
+            const int hg = sh.h[g];
+#pragma unroll
+            for (int l = 0; l < DMAX; ++l)
+                if (l == hg) m[l] += q;
+        }
+        for (int l = 0; l < L.D; ++l) L.M[static_cast<int64_t>(k) * L.D + l] = m[l];
+    }
+    __syncthreads();
+}
+
+// Exchange graph over neurons with index > lo: sh.w[a][b] = packed
+// (max gain of moving such a neuron from a to b, lowest index among ties).
+__device__ void exchange_graph(const Layer& L, Shared& sh, int lo) {
+    if (threadIdx.x < DMAX * DMAX) sh.w[threadIdx.x / DMAX][threadIdx.x % DMAX] = 0;
+    __syncthreads();
+    for (int a = 0; a < L.D; ++a) {
+        uint64_t best[DMAX];
+#pragma unroll
+        for (int b = 0; b < DMAX; ++b) best[b] = 0;
+        for (int k = threadIdx.x; k < L.N; k += kThreads) {
+            if (k <= lo || L.nu[k] != a) continue;
+            const int64_t* mk = L.M + static_cast<int64_t>(k) * L.D;
+            const int64_t ma = mk[a];
+#pragma unroll
+            for (int b = 0; b < DMAX; ++b)
+                if (b < L.D && b != a) {
+                    const uint64_t key = pack_gain(mk[b] - ma, k);
+                    best[b] = key > best[b] ? key : best[b];
+                }
+        }
+#pragma unroll
+        for (int b = 0; b < DMAX; ++b)
+            if (b < L.D && b != a) {
+                const uint64_t r = warp_max_u64(best[b]);
+                if ((threadIdx.x & 31) == 0 && r) atomicMax(reinterpret_cast<unsigned long long*>(&sh.w[a][b]), r);
+            }
+    }
+    __syncthreads();
+}
+
+__device__ void count_devices(const Layer& L, Shared& sh) {
+    if (threadIdx.x < DMAX) sh.count[threadIdx.x] = 0;
+    __syncthreads();
+    for (int k = threadIdx.x; k < L.N; k += kThreads) atomicAdd(&sh.count[L.nu[k]], 1);
+    __syncthreads();
+}
+
+// Best device of neuron k at prices pi (lowest index on ties).
+__device__ __forceinline__ int best_device(const Layer& L, const Shared& sh, int k) {
+    const int64_t* mk = L.M + static_cast<int64_t>(k) * L.D;
+    int best = 0;
+    int64_t bv = mk[0] - sh.pi[0];
+    for (int l = 1; l < L.D; ++l) {
+        const int64_t v = mk[l] - sh.pi[l];
+        if (v > bv) bv = v, best = l;
+    }
+    return best;
+}
+
+// ------------------------------------------------------------ neuron steps --
+
+__device__ void neuron_step_d2(const Layer& L, Shared& sh) {
+    const int64_t* M = L.M;
+    auto key = [M](int k) -> uint64_t { return pack_gain(M[2 * k] - M[2 * k + 1], k); };
+    const uint64_t tau = block_select_desc(L.N, L.cap, key, sh);
+    for (int k = threadIdx.x; k < L.N; k += kThreads) L.nu[k] = key(k) >= tau ? 0 : 1;
+    __syncthreads();
+}
+
+// Thread 0: max-gain path by Bellman-Ford over the D devices, from the devices
+// in `src` (dist 0) and relaxing the exchange graph sh.w.  Returns pred[].
+__device__ void bellman_ford(const Layer& L, const Shared& sh, unsigned src, int64_t* dist, int* pred) {
+    for (int a = 0; a < L.D; ++a) {
+        dist[a] = (src >> a) & 1u ? 0 : kNegInf;
+        pred[a] = -1;
+    }
+    for (int round = 0; round < L.D - 1; ++round)
+        for (int a = 0; a < L.D; ++a) {
+            if (dist[a] == kNegInf) continue;
+            for (int b = 0; b < L.D; ++b) {
+                if (b == a || sh.w[a][b] == 0) continue;
+                const int64_t nd = dist[a] + gain_of(sh.w[a][b]);
+                if (nd > dist[b]) dist[b] = nd, pred[b] = a;
+            }
+        }
+}
+
+// Thread 0: move the best neuron of each edge of the path ending at `end`.
+__device__ bool apply_path(const Layer& L, const Shared& sh, const int* pred, int end) {
+    int v = end, steps = 0;
+    while (pred[v] >= 0) {
+        if (++steps > L.D) return false;
+        const int a = pred[v];
+        L.nu[index_of(sh.w[a][v])] = v;
+        v = a;
+    }
+    return true;
+}
+
+__device__ void neuron_step_general(const Layer& L, Shared& sh) {
+    const int N = L.N, D = L.D, cap = L.cap;
+    // (a) price sweeps
+    for (int sweep = 0; sweep < 3; ++sweep) {
+        if (threadIdx.x < DMAX) sh.count[threadIdx.x] = 0;
+        __syncthreads();
+        for (int k = threadIdx.x; k < N; k += kThreads) atomicAdd(&sh.count[best_device(L, sh, k)], 1);
+        __syncthreads();
+        int excess = 0;
+        for (int l = 0; l < D; ++l) excess += sh.count[l] > cap ? sh.count[l] - cap : 0;
+        if (excess <= 2 * D) break;
+        for (int l = 0; l < D; ++l) {
+            const int64_t* M = L.M;
+            const int64_t* pi = sh.pi;
+            auto key = [M, pi, l, D](int k) -> uint64_t {
+                const int64_t* mk = M + static_cast<int64_t>(k) * D;
+                int64_t alt = kNegInf;
+                for (int m = 0; m < D; ++m)
+                    if (m != l) alt = (mk[m] - pi[m]) > alt ? (mk[m] - pi[m]) : alt;
+                const int64_t v = mk[l] - alt;
+                return static_cast<uint64_t>(v) ^ (1ull << 63);
+            };
+            const uint64_t t = block_select_desc(N, cap + 1, key, sh);
+            if (threadIdx.x == 0) sh.pi[l] = static_cast<int64_t>(t ^ (1ull << 63));
+            __syncthreads();
+        }
+    }
+    // (b) assignment at the current prices
+    for (int k = threadIdx.x; k < N; k += kThreads) L.nu[k] = best_device(L, sh, k);
+    __syncthreads();
+    count_devices(L, sh);
+    // (c) successive shortest paths until balanced
+    for (int aug = 0; aug < 4 * N + 16; ++aug) {
+        if (threadIdx.x == 0) {
+            int ex = 0;
+            for (int l = 0; l < D; ++l) ex += sh.count[l] > cap ? 1 : 0;
+            sh.flag = ex;
+        }
+        __syncthreads();
+        if (sh.flag == 0) break;
+        exchange_graph(L, sh, -1);
+        if (threadIdx.x == 0) {
+            unsigned src = 0;
+            for (int l = 0; l < D; ++l)
+                if (sh.count[l] > cap) src |= 1u << l;
+            int64_t dist[DMAX];
+            int pred[DMAX];
+            bellman_ford(L, sh, src, dist, pred);
+            int e = -1;
+            for (int l = 0; l < D; ++l)
+                if (sh.count[l] < cap && dist[l] != kNegInf && (e < 0 || dist[l] > dist[e])) e = l;
+            int s = e;
+            for (int steps = 0; e >= 0 && pred[s] >= 0 && steps <= D; ++steps) s = pred[s];
+            if (e < 0 || !apply_path(L, sh, pred, e)) {
+                sh.status = DTP_ERR_NOT_CONVERGED;
+            } else {
+                sh.count[s] -= 1;
+                sh.count[e] += 1;
+            }
+        }
+        __syncthreads();
+        if (sh.status != DTP_OK) return;
+    }
+    if (threadIdx.x == 0)
+        for (int l = 0; l < D; ++l)
+            if (sh.count[l] != cap) sh.status = DTP_ERR_NOT_CONVERGED;
+    __syncthreads();
+    if (sh.status != DTP_OK) return;
+
+    // (d) lexicographically smallest optimum
+    int kstart = 0;
+    for (int round = 0; round < N + 1; ++round) {
+        exchange_graph(L, sh, -1);
+        if (threadIdx.x == 0) {
+            for (int a = 0; a < D; ++a)
+                for (int b = 0; b < D; ++b)
+                    sh.P[a][b] = (a == b) ? 0 : (sh.w[a][b] ? gain_of(sh.w[a][b]) : kNegInf);
+            for (int c = 0; c < D; ++c)
+                for (int a = 0; a < D; ++a)
+                    for (int b = 0; b < D; ++b)
+                        if (sh.P[a][c] != kNegInf && sh.P[c][b] != kNegInf && sh.P[a][c] + sh.P[c][b] > sh.P[a][b])
+                            sh.P[a][b] = sh.P[a][c] + sh.P[c][b];
+            for (int a = 0; a < D; ++a)
+                if (sh.P[a][a] > 0) sh.status = DTP_ERR_NOT_CONVERGED;  // a positive cycle: not optimal
+            // prices for the next neuron step: longest paths from a zero root
+            for (int a = 0; a < D; ++a) sh.pi[a] = 0;
+            for (int a = 0; a < D; ++a)
+                for (int b = 0; b < D; ++b)
+                    if (sh.P[a][b] != kNegInf && sh.P[a][b] > sh.pi[b]) sh.pi[b] = sh.P[a][b];
+        }
+        __syncthreads();
+        if (sh.status != DTP_OK) return;
+        int cand = N;
+        for (int k = kstart + static_cast<int>(threadIdx.x); k < N; k += kThreads) {
+            const int t = L.nu[k];
+            const int64_t* mk = L.M + static_cast<int64_t>(k) * D;
+            for (int l = 0; l < t; ++l)
+                if (sh.P[l][t] != kNegInf && mk[l] - mk[t] + sh.P[l][t] == 0) { cand = k; break; }
+            if (cand < N) break;
+        }
+        const int kstar = block_min_int(cand, sh);
+        if (kstar >= N) break;
+        exchange_graph(L, sh, kstar);
+        if (threadIdx.x == 0) {
+            const int t = L.nu[kstar];
+            const int64_t* mk = L.M + static_cast<int64_t>(kstar) * D;
+            for (int l = 0; l < t; ++l) {
+                int64_t dist[DMAX];
+                int pred[DMAX];
+                bellman_ford(L, sh, 1u << l, dist, pred);
+                if (dist[t] != kNegInf && mk[l] - mk[t] + dist[t] == 0) {
+                    if (!apply_path(L, sh, pred, t)) sh.status = DTP_ERR_NOT_CONVERGED;
+                    L.nu[kstar] = l;
+                    break;
+                }
+            }
+        }
+        __syncthreads();
+        if (sh.status != DTP_OK) return;
+        kstart = kstar + 1;
+    }
+}
+
+// --------------------------------------------------------------- head step --
+
+__device__ void unrank_partition(int64_t idx, int G, int D, int* h) {
+    int cnt[DMAX];
+    for (int l = 0; l < D; ++l) cnt[l] = G / D;
+    uint64_t fact[GMAX + 1];
+    fact[0] = 1;
+    for (int i = 1; i <= G; ++i) fact[i] = fact[i - 1] * static_cast<uint64_t>(i);
+    for (int g = 0; g < G; ++g) {
+        const int rem = G - g - 1;
+        for (int l = 0; l < D; ++l) {
+            if (cnt[l] == 0) continue;
+            cnt[l] -= 1;
+            uint64_t ways = fact[rem];
+            for (int m = 0; m < D; ++m) ways /= fact[cnt[m]];
+            if (static_cast<uint64_t>(idx) < ways) {
+                h[g] = l;
+                break;
+            }
+            idx -= static_cast<int64_t>(ways);
+            cnt[l] += 1;
+        }
+    }
+}
+
+__device__ bool next_partition(int* h, int G) {
+    int i = G - 2;
+    while (i >= 0 && h[i] >= h[i + 1]) --i;
+    if (i < 0) return false;
+    int j = G - 1;
+    while (h[j] <= h[i]) --j;
+    int t = h[i]; h[i] = h[j]; h[j] = t;
+    for (int a = i + 1, b = G - 1; a < b; ++a, --b) t = h[a], h[a] = h[b], h[b] = t;
+    return true;
+}
+
+__device__ void head_step(const Layer& L, Shared& sh, int64_t n_parts) {
+    const int G = L.G, D = L.D;
+    if (threadIdx.x < GMAX * DMAX) sh.B[threadIdx.x] = 0;
+    __syncthreads();
+    for (int g = 0; g < G; ++g) {
+        int64_t acc[DMAX];
+#pragma unroll
+        for (int l = 0; l < DMAX; ++l) acc[l] = 0;
+        for (int k = threadIdx.x; k < L.N; k += kThreads) {
+            const int64_t q = quantize(L.A[static_cast<int64_t>(g) * L.N + k], L.e);
+            const int l0 = L.nu[k];
+#pragma unroll
+            for (int l = 0; l < DMAX; ++l)
+                if (l == l0) acc[l] += q;
+        }
+#pragma unroll
+        for (int l = 0; l < DMAX; ++l)
+            if (l < D) {
+                const int64_t s = warp_sum_i64(acc[l]);
+                if ((threadIdx.x & 31) == 0 && s)
+                    atomicAdd(reinterpret_cast<unsigned long long*>(&sh.B[g * D + l]), static_cast<unsigned long long>(s));
+            }
+    }
+    __syncthreads();
+    const int64_t lo = n_parts * threadIdx.x / kThreads;
+    const int64_t hi = n_parts * (threadIdx.x + 1) / kThreads;
+    int64_t best = kNegInf;
+    int64_t best_idx = n_parts;
+    if (lo < hi) {
+        int hh[GMAX];
+        unrank_partition(lo, G, D, hh);
+        for (int64_t idx = lo; idx < hi; ++idx) {
+            int64_t s = 0;
+            for (int g = 0; g < G; ++g) s += sh.B[g * D + hh[g]];
+            if (s > best) best = s, best_idx = idx;
+            if (idx + 1 < hi) next_partition(hh, G);
+        }
+    }
+    const int64_t bmax = block_max_i64(best, sh);
+    const int bidx = block_min_int(best == bmax ? static_cast<int>(best_idx) : 0x7FFFFFFF, sh);
+    if (threadIdx.x == 0) {
+        unrank_partition(bidx, G, D, sh.h);
+        sh.J = bmax;
+    }
+    __syncthreads();
+}
+
+// ------------------------------------------------------------------ kernel --
+
+__global__ void __launch_bounds__(kThreads, 1)
+search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, int64_t n_parts,
+              int32_t* __restrict__ head_out, int32_t* __restrict__ nu_out, int64_t* __restrict__ score_q_out,
+              double* __restrict__ score_out, int32_t* __restrict__ iters_out, int* __restrict__ status_out,
+              uint8_t* __restrict__ gbuf, size_t per_layer, int use_smem) {
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ Shared sh;
+    const int layer = blockIdx.x;
+    uint8_t* buf = use_smem ? dsm : gbuf + static_cast<size_t>(layer) * per_layer;
+    Layer L;
+    L.A = A_all + static_cast<int64_t>(layer) * G * N;
+    L.G = G;
+    L.N = N;
+    L.D = D;
+    L.cap = N / D;
+    L.M = reinterpret_cast<int64_t*>(buf);
+    L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * D * sizeof(int64_t));
+
+    if (threadIdx.x == 0) {
+        sh.status = DTP_OK;
+        for (int l = 0; l < DMAX; ++l) sh.pi[l] = 0;
+    }
+    // validity and the fixed-point exponent
+    uint32_t amax_bits = 0;
+    int bad = 0;
+    for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) {
+        const float a = L.A[i];
+        if (!(a >= 0.0f) || isinf(a)) bad = 1;
+        else amax_bits = max(amax_bits, __float_as_uint(a));
+    }
+    bad = __syncthreads_or(bad);
+    const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
+    if (bad) {
+        if (threadIdx.x == 0) status_out[layer] = DTP_ERR_ARG;
+        return;
+    }
+    const float amax = __uint_as_float(static_cast<uint32_t>(amax_all));
+    int e = 0;
+    if (amax > 0.0f) frexpf(amax, &e);
+    L.e = e;
+    int64_t part = 0;
+    for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) part += quantize(L.A[i], e);
+    const int64_t total = block_sum_i64(part, sh);
+    if (threadIdx.x < G) sh.h[threadIdx.x] = (threadIdx.x * D) / G;
+    if (threadIdx.x == 0) sh.Jprev = -1;
+    __syncthreads();
+
+    int done = 0;
+    for (int it = 0; it < iters; ++it) {
+        build_gain(L, sh);
+        if (D == 2) neuron_step_d2(L, sh);
+        else neuron_step_general(L, sh);
+        if (sh.status != DTP_OK) break;
+        head_step(L, sh, n_parts);
+        done = it + 1;
+        const bool stop = sh.J <= sh.Jprev;
+        __syncthreads();
+        if (threadIdx.x == 0) sh.Jprev = sh.J;
+        __syncthreads();
+        if (stop) break;
+    }
+    __syncthreads();
+    if (sh.status != DTP_OK) {
+        if (threadIdx.x == 0) status_out[layer] = sh.status;
+        return;
+    }
+    for (int k = threadIdx.x; k < N; k += kThreads) nu_out[static_cast<int64_t>(layer) * N + k] = L.nu[k];
+    if (threadIdx.x < G) head_out[static_cast<int64_t>(layer) * G + threadIdx.x] = sh.h[threadIdx.x];
+    if (threadIdx.x == 0) {
+        score_q_out[layer] = sh.J;
+        score_out[layer] = total > 0 ? static_cast<double>(sh.J) / static_cast<double>(total) : 0.0;
+        iters_out[layer] = done;
+        status_out[layer] = DTP_OK;
+    }
+}
+
+// --------------------------------------------------------------------- host --
+
+int64_t partition_count(int G, int D) {
+    // G! / ((G/D)!)^D
+    double f[GMAX + 1];
+    f[0] = 1.0;
+    for (int i = 1; i <= GMAX; ++i) f[i] = f[i - 1] * i;
+    double c = f[G];
+    for (int l = 0; l < D; ++l) c /= f[G / D];
+    return static_cast<int64_t>(c + 0.5);
+}
+
+static size_t per_layer_bytes(int N, int D) {
+    return align_up(static_cast<size_t>(N) * D * sizeof(int64_t) + static_cast<size_t>(N) * sizeof(int32_t), 256);
+}
+
+static bool fits_smem(int N, int D) { return per_layer_bytes(N, D) <= kSmemBudget; }
+
+size_t workspace_bytes(int layers, int G, int N, int D) {
+    (void)G;
+    size_t b = kWorkspaceHeader + align_up(static_cast<size_t>(layers) * sizeof(int), 256);
+    if (!fits_smem(N, D)) b += static_cast<size_t>(layers) * per_layer_bytes(N, D);
+    return b;
+}
+
+int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* head, int32_t* nu, int64_t* score_q,
+           double* score, int32_t* iters_done, void* workspace, cudaStream_t stream) {
+    uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+    int* status = reinterpret_cast<int*>(ws + kWorkspaceHeader);
+    uint8_t* gbuf = ws + kWorkspaceHeader + align_up(static_cast<size_t>(layers) * sizeof(int), 256);
+    const bool smem = fits_smem(N, D);
+    const size_t dyn = smem ? per_layer_bytes(N, D) : 0;
+    DTP_CUDA_TRY(cudaFuncSetAttribute(search_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kSmemBudget)));
+    // sentinel 0xFEFEFEFE: a layer whose kernel never reported reads as a CUDA failure
+    DTP_CUDA_TRY(cudaMemsetAsync(status, 0xFE, static_cast<size_t>(layers) * sizeof(int), stream));
+    search_kernel<<<layers, kThreads, dyn, stream>>>(A, G, N, D, iters, partition_count(G, D), head, nu, score_q,
+                                                      score, iters_done, status, gbuf, per_layer_bytes(N, D),
+                                                      smem ? 1 : 0);
+    DTP_CUDA_TRY(cudaGetLastError());
+    int* host = static_cast<int*>(malloc(static_cast<size_t>(layers) * sizeof(int)));
+    if (!host) return DTP_ERR_CUDA;
+    cudaError_t err = cudaMemcpyAsync(host, status, static_cast<size_t>(layers) * sizeof(int),
+                                      cudaMemcpyDeviceToHost, stream);
+    if (err == cudaSuccess) err = cudaStreamSynchronize(stream);
+    int rc = DTP_OK;
+    if (err != cudaSuccess) rc = DTP_ERR_CUDA;
+    for (int i = 0; rc == DTP_OK && i < layers; ++i) {
+        const int st = host[i];
+        if (st == DTP_OK) continue;
+        rc = (st == DTP_ERR_ARG || st == DTP_ERR_NOT_CONVERGED) ? st : DTP_ERR_CUDA;
+    }
+    free(host);
+    return rc;
+}
+
+}  // namespace search
+}  // namespace dtp

@@ -1,0 +1,199 @@
+"""ctypes binding of libdtp.so (include/dtp.h), argument marshalling only.
+
+Every computation runs in the library's CUDA kernels; this module checks
+tensor shapes, dtypes and devices, allocates caller-side outputs and
+workspaces with PyTorch, and passes raw device pointers plus the current CUDA
+stream.  It raises if the library was not built: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libdtp.so")
+
+DTP_OK = 0
+DTP_ERR_ARG = -1
+DTP_ERR_CUDA = -2
+DTP_ERR_NOT_CONVERGED = -3
+DTP_ERR_UNSUPPORTED = -4
+DTP_ERR_WORKSPACE = -5
+DTP_BF16 = 0
+DTP_F32 = 1
+
+_lib = None
+
+_vp = ctypes.c_void_p
+_i64 = ctypes.c_int64
+_i32 = ctypes.c_int
+_sz = ctypes.c_size_t
+
+
+class DTPError(RuntimeError):
+    """A libdtp call returned a non-zero dtp_status."""
+
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn}: {status_string(status)} ({status})")
+
+
+def lib():
+    """Load libdtp.so (built by ``paper_2609_13846_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with `python -m paper_2609_13846_gb300.build`")
+    L = ctypes.CDLL(LIB_PATH)
+    L.dtp_version.restype = _i32
+    L.dtp_status_string.argtypes = [_i32]
+    L.dtp_status_string.restype = ctypes.c_char_p
+    L.dtp_affinity_workspace_size.argtypes = [_i64, _i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_affinity_accumulate.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
+    L.dtp_affinity_finalize.argtypes = [_vp, _i32, _i32, _i64, _vp, _vp]
+    L.dtp_down_sqnorm.argtypes = [_vp, _i32, _i32, _i32, _vp, _vp]
+    L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
+    L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+    L.dtp_search_layout_batched.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                            _vp]
+    for fn in ("dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_finalize",
+               "dtp_down_sqnorm", "dtp_workspace_status", "dtp_search_workspace_size", "dtp_search_layout",
+               "dtp_search_layout_batched"):
+        getattr(L, fn).restype = _i32
+    _lib = L
+    return L
+
+
+def status_string(status: int) -> str:
+    return lib().dtp_status_string(int(status)).decode()
+
+
+def _check(fn: str, status: int):
+    if status != DTP_OK:
+        raise DTPError(fn, status)
+
+
+def _stream(stream=None) -> int:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return int(s.cuda_stream)
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return DTP_BF16
+    if t.dtype == torch.float32:
+        return DTP_F32
+    raise TypeError(f"unsupported dtype {t.dtype}; use bfloat16 or float32")
+
+
+def affinity_workspace_size(T: int, d: int, H_kv: int, N: int, dtype: int) -> int:
+    n = _sz(0)
+    _check("dtp_affinity_workspace_size", lib().dtp_affinity_workspace_size(T, d, H_kv, N, dtype, ctypes.byref(n)))
+    return n.value
+
+
+def affinity_workspace(T: int, d: int, H_kv: int, N: int, dtype: int, device) -> torch.Tensor:
+    """A device workspace tensor sized for these arguments."""
+    return torch.empty(affinity_workspace_size(T, d, H_kv, N, dtype), dtype=torch.uint8, device=device)
+
+
+def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
+                        A: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                        stream=None) -> torch.Tensor:
+    """A[h,k] += sum_t Delta_{t,h,k}^2 (Sec. 3); returns A [H_kv, N] fp32 on X's device.
+
+    X [T,d], C [H_kv,T,d], W_gate/W_up [N,d]: contiguous CUDA tensors, all bf16
+    or all fp32.  ``A`` is accumulated into (a zero tensor is made if None).
+    """
+    for name, t in (("X", X), ("C", C), ("W_gate", W_gate), ("W_up", W_up)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    if not (X.dtype == C.dtype == W_gate.dtype == W_up.dtype):
+        raise TypeError("X, C, W_gate and W_up must share one dtype")
+    T, d = X.shape
+    H = C.shape[0]
+    N = W_gate.shape[0]
+    if C.shape != (H, T, d) or W_gate.shape != (N, d) or W_up.shape != (N, d):
+        raise ValueError("shapes must be X [T,d], C [H,T,d], W_gate [N,d], W_up [N,d]")
+    code = _dtype_code(X)
+    if A is None:
+        A = torch.zeros((H, N), dtype=torch.float32, device=X.device)
+    if A.shape != (H, N) or A.dtype != torch.float32 or not A.is_contiguous() or A.device != X.device:
+        raise ValueError("A must be a contiguous fp32 [H_kv, N] tensor on X's device")
+    if workspace is None:
+        workspace = affinity_workspace(T, d, H, N, code, X.device)
+    st = lib().dtp_affinity_accumulate(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, code, _ptr(A),
+                                       _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_affinity_accumulate", st)
+    return A
+
+
+def workspace_status(workspace: torch.Tensor, stream=None) -> int:
+    """Synchronise and read the workspace status word (DTP_OK or DTP_ERR_NOT_CONVERGED)."""
+    return int(lib().dtp_workspace_status(_ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def affinity_finalize(A: torch.Tensor, T_total: int, wd_sqnorm: torch.Tensor | None = None, stream=None):
+    """In place: A *= wd_sqnorm[k] / T_total (Sec. 3 E_t mean and ||w^d_k||^2)."""
+    H, N = A.shape
+    if wd_sqnorm is not None and (wd_sqnorm.shape != (N,) or wd_sqnorm.dtype != torch.float32):
+        raise ValueError("wd_sqnorm must be fp32 [N]")
+    _check("dtp_affinity_finalize",
+           lib().dtp_affinity_finalize(_ptr(A), H, N, int(T_total), _ptr(wd_sqnorm), _stream(stream)))
+    return A
+
+
+def down_sqnorm(W_down: torch.Tensor, stream=None) -> torch.Tensor:
+    """||w^d_k||^2 for W_down [d, N] (nn.Linear [out=d, in=N]) -> fp32 [N]."""
+    d, N = W_down.shape
+    out = torch.empty(N, dtype=torch.float32, device=W_down.device)
+    _check("dtp_down_sqnorm",
+           lib().dtp_down_sqnorm(_ptr(W_down), d, N, _dtype_code(W_down), _ptr(out), _stream(stream)))
+    return out
+
+
+def search_workspace_size(layers: int, H_kv: int, N: int, D: int) -> int:
+    n = _sz(0)
+    _check("dtp_search_workspace_size", lib().dtp_search_workspace_size(layers, H_kv, N, D, ctypes.byref(n)))
+    return n.value
+
+
+def search_layout_batched(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor | None = None,
+                          stream=None) -> dict:
+    """Coordinate ascent on each layer of A [L, H_kv, N] (Sec. 3 'Optimiser').
+
+    Returns dict of device tensors: h [L,H_kv] int32, nu [L,N] int32,
+    score_q [L] int64, score [L] float64, iters_done [L] int32.  Synchronous.
+    """
+    if A.dim() == 2:
+        A = A.unsqueeze(0)
+    if A.dtype != torch.float32 or not A.is_cuda or not A.is_contiguous():
+        raise ValueError("A must be a contiguous fp32 CUDA tensor [L, H_kv, N]")
+    Lyr, H, N = A.shape
+    dev = A.device
+    out = dict(h=torch.empty((Lyr, H), dtype=torch.int32, device=dev),
+               nu=torch.empty((Lyr, N), dtype=torch.int32, device=dev),
+               score_q=torch.empty(Lyr, dtype=torch.int64, device=dev),
+               score=torch.empty(Lyr, dtype=torch.float64, device=dev),
+               iters_done=torch.empty(Lyr, dtype=torch.int32, device=dev))
+    if workspace is None:
+        workspace = torch.empty(search_workspace_size(Lyr, H, N, D), dtype=torch.uint8, device=dev)
+    st = lib().dtp_search_layout_batched(_ptr(A), Lyr, H, N, D, iters, _ptr(out["h"]), _ptr(out["nu"]),
+                                         _ptr(out["score_q"]), _ptr(out["score"]), _ptr(out["iters_done"]),
+                                         _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_search_layout_batched", st)
+    return out
+
+
+def search_layout(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor | None = None, stream=None) -> dict:
+    """Coordinate ascent on one layer's A [H_kv, N]; tensors as in search_layout_batched, unbatched."""
+    r = search_layout_batched(A.unsqueeze(0) if A.dim() == 2 else A, D, iters, workspace, stream)
+    return {k: v[0] for k, v in r.items()}

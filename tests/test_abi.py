@@ -1,0 +1,100 @@
+"""The C-ABI library loads and exports every entry point include/dtp.h declares;
+host-side argument validation rejects bad calls before any launch (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "dtp.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_13846_gb300 import build, dtp
+    build.build()
+    return dtp.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(dtp_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("dtp_affinity_accumulate", "dtp_search_layout", "dtp_search_layout_batched",
+                     "dtp_affinity_workspace_size", "dtp_search_workspace_size", "dtp_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), f"{name} not exported by libdtp.so"
+
+
+def test_no_symbol_outside_header_is_extern_c(lib):
+    """The library has no extra dtp_* C symbols beyond the header's."""
+    import subprocess
+    from paper_2609_13846_gb300 import dtp
+    out = subprocess.run(["nm", "-D", "--defined-only", dtp.LIB_PATH], capture_output=True, text=True).stdout
+    exported = sorted({m for m in re.findall(r"\bT (dtp_[a-z0-9_]+)\b", out)})
+    assert exported == declared_functions()
+
+
+def test_version_and_status_strings(lib):
+    from paper_2609_13846_gb300 import dtp
+    assert lib.dtp_version() >= 100
+    assert dtp.status_string(0) == "ok"
+    assert "argument" in dtp.status_string(-1)
+    assert dtp.status_string(12345) == "unknown status"
+
+
+def test_workspace_size_queries(lib):
+    from paper_2609_13846_gb300 import dtp
+    n = dtp.affinity_workspace_size(16384, 1024, 8, 3072, dtp.DTP_BF16)
+    assert n >= 256 + 128 * 24 * 2 * 8 * 128 * 4
+    assert dtp.affinity_workspace_size(256, 64, 2, 128, dtp.DTP_F32) > 256
+    assert dtp.search_workspace_size(28, 8, 3072, 4) >= 256
+    # a layer that does not fit in shared memory gets a global buffer
+    assert dtp.search_workspace_size(1, 8, 14336, 8) > 14336 * 8 * 8
+
+
+@pytest.mark.parametrize("args", [
+    (-1, 64, 2, 128, 0), (16, 12, 2, 128, 0), (16, 64, 0, 128, 0), (16, 64, 17, 128, 0),
+    (16, 64, 2, 0, 0), (16, 64, 2, 128, 7)])
+def test_affinity_size_query_rejects_bad_sizes(lib, args):
+    n = ctypes.c_size_t(0)
+    assert lib.dtp_affinity_workspace_size(*args, ctypes.byref(n)) == -1
+
+
+def test_affinity_rejects_null_and_misaligned_before_launch(lib):
+    vp = ctypes.c_void_p
+    ok = vp(1 << 20)
+    bad = vp((1 << 20) + 2)
+    # null input
+    assert lib.dtp_affinity_accumulate(None, ok, ok, ok, 16, 64, 2, 128, 0, ok, ok, 1 << 30, None) == -1
+    # misaligned weight
+    assert lib.dtp_affinity_accumulate(ok, ok, bad, ok, 16, 64, 2, 128, 0, ok, ok, 1 << 30, None) == -1
+    # workspace too small
+    assert lib.dtp_affinity_accumulate(ok, ok, ok, ok, 16, 64, 2, 128, 0, ok, ok, 8, None) == -5
+    # d not a multiple of 8
+    assert lib.dtp_affinity_accumulate(ok, ok, ok, ok, 16, 60, 2, 128, 0, ok, ok, 1 << 30, None) == -1
+
+
+@pytest.mark.parametrize("layers,H,N,D,iters", [
+    (1, 8, 3072, 3, 10), (1, 8, 3071, 2, 10), (1, 8, 3072, 16, 10), (1, 8, 3072, 1, 10),
+    (0, 8, 3072, 2, 10), (1, 8, 3072, 2, 0), (1, 32, 64, 2, 1), (1, 8, 1 << 19, 2, 1)])
+def test_search_rejects_bad_sizes(lib, layers, H, N, D, iters):
+    vp = ctypes.c_void_p
+    ok = vp(1 << 20)
+    st = lib.dtp_search_layout_batched(ok, layers, H, N, D, iters, ok, ok, ok, ok, ok, ok, 1 << 30, None)
+    assert st == -1
+
+
+def test_search_rejects_missing_workspace(lib):
+    vp = ctypes.c_void_p
+    ok = vp(1 << 20)
+    assert lib.dtp_search_layout(ok, 8, 64, 2, 3, ok, ok, ok, ok, ok, None, 0, None) == -5

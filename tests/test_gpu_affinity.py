@@ -1,0 +1,145 @@
+"""GPU parity of the first-order affinity (Sec. 3 "Affinity scores") against the fp64 oracle.
+
+Tolerances (relative Frobenius error of A): 5e-3 for bf16 operands (tcgen05
+path), 1e-5 for the fp32 mode.  The inputs are the same bf16/fp32 values on
+both sides, so the error budget is fp32 accumulation and the fp32 epilogue.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_13846_gb300 import dtp, synth
+
+pytestmark = pytest.mark.gpu
+
+BF16_TOL = 5e-3
+F32_TOL = 1e-5
+DEV = "cuda:0"
+
+
+def _rel_fro(a, b):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def _oracle(L, rows=None):
+    X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
+    if rows is not None:
+        Wg, Wu = Wg[rows], Wu[rows]
+    return oracle.affinity_fo(X, C, Wg, Wu)
+
+
+def _gpu(L, A=None):
+    g = {k: v.to(DEV) for k, v in L.items()}
+    out = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"], A=A)
+    torch.cuda.synchronize()
+    return out
+
+
+def test_tiny_workload_fp32_mode():
+    """The tiny calibration workload (d=64, G=2, N=128, T=256) in fp32 mode: <= 1e-5."""
+    L = synth.make_workload_layer(synth.WORKLOADS["tiny"])
+    A = _gpu(L).cpu().numpy()
+    assert _rel_fro(A, _oracle(L)) <= F32_TOL
+
+
+def test_tiny_workload_bf16_mode():
+    L = synth.make_workload_layer(synth.WORKLOADS["tiny"])
+    Lb = {k: v.to(torch.bfloat16) for k, v in L.items()}
+    A = _gpu(Lb).cpu().numpy()
+    assert _rel_fro(A, _oracle(Lb)) <= BF16_TOL
+
+
+@pytest.mark.parametrize("d,G,N,T", [
+    (328, 3, 300, 333),     # ragged in every dimension, several tiles of each
+    (1024, 8, 384, 384),    # Qwen-like d and G, 3 neuron tiles x 3 token chunks
+    (64, 1, 1, 1),          # single head, neuron and token
+    (8, 2, 130, 129),       # smallest d (one 16-byte row), ragged tiles
+    (136, 16, 200, 77),     # the largest supported head count
+])
+def test_bf16_parity_ragged(d, G, N, T):
+    L = synth.make_layer(d, G, N, T, seed=d + G + N + T, dtype="bf16", outliers=d >= 64)
+    A = _gpu(L).cpu().numpy()
+    err = _rel_fro(A, _oracle(L))
+    assert err <= BF16_TOL, err
+    # elementwise: every entry within a loose relative bound of the fp64 value
+    ref = _oracle(L)
+    assert np.all(np.abs(A - ref) <= 2e-2 * np.abs(ref) + 1e-6 * np.abs(ref).max())
+
+
+@pytest.mark.parametrize("d,G,N,T", [(328, 3, 300, 333), (64, 2, 65, 70)])
+def test_fp32_parity_ragged(d, G, N, T):
+    L = synth.make_layer(d, G, N, T, seed=3, dtype="f32", outliers=True)
+    A = _gpu(L).cpu().numpy()
+    assert _rel_fro(A, _oracle(L)) <= F32_TOL
+
+
+def test_zero_tokens_is_a_noop():
+    L = synth.make_layer(64, 2, 32, 8, seed=1, dtype="bf16")
+    g = {k: v.to(DEV) for k, v in L.items()}
+    A = torch.full((2, 32), 3.0, device=DEV)
+    dtp.affinity_accumulate(g["X"][:0].contiguous(), g["C"][:, :0].contiguous(), g["W_gate"], g["W_up"], A=A)
+    torch.cuda.synchronize()
+    assert torch.all(A == 3.0)
+
+
+def test_accumulates_over_token_chunks():
+    """A is accumulated, so streaming token chunks equals one call on all tokens (Sec. 3: E_t over tokens)."""
+    L = synth.make_layer(256, 4, 256, 600, seed=9, dtype="bf16")
+    full = _gpu(L)
+    A = torch.zeros_like(full)
+    for lo, hi in ((0, 128), (128, 333), (333, 600)):
+        part = {"X": L["X"][lo:hi].contiguous(), "C": L["C"][:, lo:hi].contiguous(),
+                "W_gate": L["W_gate"], "W_up": L["W_up"]}
+        _gpu(part, A=A)
+    assert torch.allclose(A, full, rtol=1e-5, atol=0)
+
+
+def test_deterministic():
+    L = synth.make_layer(512, 8, 384, 1024, seed=4, dtype="bf16")
+    a = _gpu(L)
+    b = _gpu(L)
+    assert torch.equal(a, b)
+
+
+def test_workspace_status_ok_and_explicit_workspace():
+    L = synth.make_layer(128, 2, 128, 256, seed=2, dtype="bf16")
+    g = {k: v.to(DEV) for k, v in L.items()}
+    ws = dtp.affinity_workspace(256, 128, 2, 128, dtp.DTP_BF16, DEV)
+    A = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"], workspace=ws)
+    assert dtp.workspace_status(ws) == dtp.DTP_OK
+    assert _rel_fro(A.cpu().numpy(), _oracle(L)) <= BF16_TOL
+
+
+def test_finalize_and_down_norm():
+    """S^{up,fo} = E_t[Delta^2] ||w^d_k||^2 (Sec. 3)."""
+    L = synth.make_layer(128, 2, 96, 200, seed=5, dtype="bf16", with_down=True)
+    A = _gpu({k: L[k] for k in ("X", "C", "W_gate", "W_up")})
+    wd = dtp.down_sqnorm(L["W_down"].to(DEV))
+    ref_wd = (L["W_down"].double() ** 2).sum(0).numpy()
+    assert np.allclose(wd.cpu().numpy(), ref_wd, rtol=1e-5)
+    dtp.affinity_finalize(A, 200, wd)
+    torch.cuda.synchronize()
+    ref = oracle.finalize(_oracle(L), 200, ref_wd)
+    assert _rel_fro(A.cpu().numpy(), ref) <= BF16_TOL
+
+
+@pytest.mark.parametrize("name", ["qwen3_0.6b_layer", "llama3.1_8b_layer"])
+def test_full_size_sampled_neurons(name):
+    """Full-size layer in the launch configuration the benchmark times; the oracle
+    computes a sample of neuron columns over all T tokens (column k of A depends
+    only on row k of the weights)."""
+    w = synth.WORKLOADS[name]
+    L = synth.make_workload_layer(w, device=DEV)
+    A = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"])
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(0)
+    cols = np.sort(rng.choice(w.N, size=6, replace=False))
+    cols = np.unique(np.concatenate([cols, [0, w.N - 1]]))
+    Lh = {k: v.cpu() for k, v in L.items()}
+    ref = _oracle(Lh, rows=cols)
+    got = A[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
+    assert _rel_fro(got, ref) <= BF16_TOL
+    assert torch.isfinite(A).all() and (A >= 0).all()

@@ -1,0 +1,99 @@
+"""GPU parity of the layout optimiser (Sec. 3 "Objective", "Optimiser") against the oracle.
+
+Both sides get the same fp32 A; the contract is bit-exact on the head
+partition h, the neuron assignment nu (lexicographically smallest optimum),
+the integer score and the iteration count.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_13846_gb300 import dtp, synth
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+def _compare(A_np, D, iters, res=None):
+    if res is None:
+        res = dtp.search_layout(torch.as_tensor(A_np, device=DEV), D, iters)
+    ref = oracle.search_layout(A_np, D, iters)
+    np.testing.assert_array_equal(res["h"].cpu().numpy(), ref["h"])
+    np.testing.assert_array_equal(res["nu"].cpu().numpy(), ref["nu"])
+    assert int(res["score_q"]) == ref["score_q"]
+    assert int(res["iters_done"]) == ref["iters_done"]
+    assert float(res["score"]) == pytest.approx(ref["score"], rel=1e-15, abs=0)
+    return ref
+
+
+@pytest.mark.parametrize("G,N,D", [(2, 128, 2), (8, 3072, 2), (8, 256, 4), (8, 3072, 4), (8, 512, 8),
+                                   (6, 96, 3), (4, 1000, 2), (16, 64, 2), (12, 120, 4), (8, 24, 8)])
+@pytest.mark.parametrize("kind", ["lognormal", "integer"])
+def test_search_matches_oracle(G, N, D, kind):
+    A = synth.make_affinity_matrix(G, N, seed=G * 1000 + N + D, kind=kind).numpy()
+    _compare(A, D, 10)
+
+
+@pytest.mark.parametrize("iters", [1, 2, 3])
+def test_iteration_cap(iters):
+    A = synth.make_affinity_matrix(8, 512, seed=77).numpy()
+    _compare(A, 4, iters)
+
+
+def test_zero_matrix_returns_contiguous_layout():
+    A = np.zeros((8, 64), dtype=np.float32)
+    ref = _compare(A, 4, 10)
+    np.testing.assert_array_equal(ref["h"], [0, 0, 1, 1, 2, 2, 3, 3])
+
+
+def test_batched_layers_match_per_layer_oracle():
+    As = np.stack([synth.make_affinity_matrix(8, 3072, seed=100 + i).numpy() for i in range(6)])
+    res = dtp.search_layout_batched(torch.as_tensor(As, device=DEV), 4, 10)
+    for i in range(6):
+        _compare(As[i], 4, 10, res={k: v[i] for k, v in res.items()})
+
+
+def test_from_gpu_affinity_tiny_workload():
+    """The tiny workload end to end: GPU affinity, then both searches on that A."""
+    L = synth.make_workload_layer(synth.WORKLOADS["tiny"], device=DEV)
+    A = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"])
+    _compare(A.cpu().numpy(), 2, 10)
+
+
+def test_full_size_qwen_d2_and_d4():
+    """Qwen3-0.6B shape (G=8, N=3072), a batch of layers from the GPU affinity pass on a token slice."""
+    w = synth.WORKLOADS["qwen3_0.6b_model"]
+    As = []
+    for layer in range(3):
+        L = synth.make_workload_layer(w, layer, T=2048, device=DEV)
+        As.append(dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"]))
+    A = torch.stack(As).contiguous()
+    for D in (2, 4):
+        res = dtp.search_layout_batched(A, D, 10)
+        An = A.cpu().numpy()
+        for i in range(A.shape[0]):
+            _compare(An[i], D, 10, res={k: v[i] for k, v in res.items()})
+
+
+def test_full_size_llama_neuron_count_d8():
+    """Llama-3.1-8B shape N=14336 (global-memory path of the search), D=8."""
+    A = synth.make_affinity_matrix(8, 14336, seed=3).numpy()
+    _compare(A, 8, 10)
+
+
+@pytest.mark.parametrize("bad", [-1.0, float("nan"), float("inf")])
+def test_invalid_entries_rejected(bad):
+    A = synth.make_affinity_matrix(8, 64, seed=1)
+    A[3, 5] = bad
+    with pytest.raises(dtp.DTPError) as e:
+        dtp.search_layout(A.to(DEV), 2, 10)
+    assert e.value.status == dtp.DTP_ERR_ARG
+
+
+def test_search_is_deterministic():
+    A = torch.as_tensor(synth.make_affinity_matrix(8, 3072, seed=5).numpy(), device=DEV)
+    a = dtp.search_layout(A, 4, 10)
+    b = dtp.search_layout(A, 4, 10)
+    for k in a:
+        assert torch.equal(a[k], b[k])
