@@ -111,6 +111,29 @@ int dtp_affinity_finalize(float* A, int H_kv, int N, int64_t T_total, const floa
 int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, void* stream);
 
 /*
+ * dtp_affinity_accumulate with DTP_BF16 for callers that cannot allocate
+ * device memory or pass a workspace (e.g. a plugin whose host application
+ * owns every device allocation, or a runtime with a fixed memory plan that
+ * must not grow after start-up).  The paper has no counterpart: this entry
+ * point only changes where the scratch lives.
+ *
+ * Same arguments, layouts, accumulation and result as dtp_affinity_accumulate
+ * (bf16 inputs only), minus the workspace.  Scratch comes from one fixed
+ * device array of 32 MiB + 256 B inside the library, present on every GPU
+ * that loads it until the process exits; the call allocates nothing.
+ *   - Limit: ceil(T/128) * ceil(N/128) * H_kv <= 32768 per call, else
+ *     DTP_ERR_WORKSPACE (stream longer inputs as token chunks; A accumulates).
+ *   - Every call shares the array and it keeps the last call's contents:
+ *     calls that overlap on the GPU race and must be serialised by the caller.
+ *   - The first call on a device looks up the array's device address with
+ *     that device current; make it before any stream capture begins.
+ * Asynchronous on `stream`.
+ */
+int dtp_affinity_accumulate_noalloc(const void* X, const void* C, const void* W_gate,
+                                    const void* W_up, int64_t T, int d, int H_kv, int N, float* A,
+                                    void* stream);
+
+/*
  * Synchronises `stream`, then reads the status word that kernels of the last
  * call using `workspace` leave in it: DTP_OK, or DTP_ERR_NOT_CONVERGED if a
  * bounded device-side wait gave up.  workspace_bytes as passed to that call.

@@ -55,12 +55,14 @@ def lib():
     L.dtp_affinity_accumulate.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
     L.dtp_affinity_finalize.argtypes = [_vp, _i32, _i32, _i64, _vp, _vp]
     L.dtp_down_sqnorm.argtypes = [_vp, _i32, _i32, _i32, _vp, _vp]
+    L.dtp_affinity_accumulate_noalloc.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_search_layout_batched.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                             _vp]
-    for fn in ("dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_finalize",
+    for fn in ("dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
+               "dtp_affinity_finalize",
                "dtp_down_sqnorm", "dtp_workspace_status", "dtp_search_workspace_size", "dtp_search_layout",
                "dtp_search_layout_batched"):
         getattr(L, fn).restype = _i32
@@ -133,6 +135,23 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
     st = lib().dtp_affinity_accumulate(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, code, _ptr(A),
                                        _ptr(workspace), workspace.numel(), _stream(stream))
     _check("dtp_affinity_accumulate", st)
+    return A
+
+
+def affinity_accumulate_noalloc(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
+                                A: torch.Tensor, stream=None) -> torch.Tensor:
+    """bf16 affinity pass that allocates nothing: scratch is the library's fixed device array.
+
+    For callers that cannot allocate device memory; the caller passes the
+    inputs and the fp32 output A [H_kv, N], which is accumulated into.  Calls
+    that overlap on the GPU share the scratch and race.
+    """
+    T, d = X.shape
+    H = C.shape[0]
+    N = W_gate.shape[0]
+    st = lib().dtp_affinity_accumulate_noalloc(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, _ptr(A),
+                                               _stream(stream))
+    _check("dtp_affinity_accumulate_noalloc", st)
     return A
 
 
