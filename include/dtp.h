@@ -119,7 +119,7 @@ int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, voi
  *
  * Same arguments, layouts, accumulation and result as dtp_affinity_accumulate
  * (bf16 inputs only), minus the workspace.  Scratch comes from one fixed
- * device array of 32 MiB + 256 B inside the library, present on every GPU
+ * device array of 16 MiB + 256 B inside the library, present on every GPU
  * that loads it until the process exits; the call allocates nothing.
  *   - Limit: ceil(T/128) * ceil(N/128) * H_kv <= 32768 per call, else
  *     DTP_ERR_WORKSPACE (stream longer inputs as token chunks; A accumulates).

@@ -33,9 +33,10 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
 }  // namespace tc
 }  // namespace dtp
 
-// 256-byte status header + 32 MiB of partial sums:
-// ceil(T/128) * ceil(N/128) * H_kv <= 32768 per call (1 KiB per token chunk, neuron tile and head).
-static constexpr size_t kNoAllocScratchBytes = dtp::kWorkspaceHeader + (size_t(32) << 20);
+// 256-byte status header + 16 MiB of partial sums (512 B per token chunk,
+// neuron tile and head): ceil(T/128) * ceil(N/128) * H_kv <= 32768 per call.
+static constexpr int64_t kNoAllocMaxUnitHeads = 32768;
+static constexpr size_t kNoAllocScratchBytes = dtp::kWorkspaceHeader + (size_t(16) << 20);
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 namespace {
@@ -72,7 +73,9 @@ extern "C" int dtp_affinity_accumulate_noalloc(const void* X, const void* C, con
     if (!dtp::aligned16(X) || !dtp::aligned16(C) || !dtp::aligned16(W_gate) || !dtp::aligned16(W_up) ||
         !dtp::aligned16(A))
         return DTP_ERR_ARG;
-    if (dtp::tc::workspace_bytes(T, d, H_kv, N) > kNoAllocScratchBytes) return DTP_ERR_WORKSPACE;
+    const int64_t unit_heads = ((T + 127) / 128) * ((static_cast<int64_t>(N) + 127) / 128) * H_kv;
+    if (unit_heads > kNoAllocMaxUnitHeads || dtp::tc::workspace_bytes(T, d, H_kv, N) > kNoAllocScratchBytes)
+        return DTP_ERR_WORKSPACE;
     void* scratch = nullptr;
     const int rc = scratch_address(&scratch);
     if (rc != DTP_OK) return rc;

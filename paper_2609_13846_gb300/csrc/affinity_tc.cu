@@ -6,31 +6,36 @@
 // with g = X W_gate^T, u = X W_up^T (the operating point) and pg = C_h W_gate^T,
 // pu = C_h W_up^T (head h's piece projected through the FFN input weights).
 //
-// Orientation.  The MMA's M dimension is the neuron (128 neurons of one tile
-// in the 128 TMEM lanes) and its N dimension is the token (a chunk of 128
-// tokens in TMEM columns).  Each epilogue thread therefore owns one neuron
-// and sums Delta^2 over tokens inside its own registers: the token reduction
-// needs no shuffles, and the T x G x N intermediate never leaves the SM.
+// MMA shape.  One tcgen05.mma per 16-wide K step computes a 128-token x
+// 256-column tile: A = 128 rows of one activation tile (X or C_h), B = the
+// neuron tile's 128 W_gate rows stacked on its 128 W_up rows, so columns
+// [0,128) of the accumulator are g (or pg) and [128,256) are u (or pu) of the
+// same 128 neurons.  The kernel is bound by the number of MMA instructions it
+// issues, so the widest single-CTA instruction (N = 256) is used.
 //
-// Work unit = (token chunk c, neuron tile j); a unit runs G+1 passes over d:
-// pass 0 multiplies the X chunk, pass 1+h the C_h chunk, each against the
-// tile's W_gate and W_up rows (two M=128, N=128 MMAs per K step sharing the
-// activation operand).  Units are dealt round-robin to a persistent grid in
+// Work unit = (token chunk c of 128 tokens, neuron tile j of 128 neurons).  A
+// unit runs G+1 passes over d: pass 0 multiplies the X chunk, pass 1+h the C_h
+// chunk.  Units are dealt round-robin to a persistent grid in
 // token-chunk-major order, so the CTAs in flight share a handful of token
 // chunks in L2 while all weights stay L2-resident.
 //
-// TMEM (512 columns x 128 lanes, fp32):
-//     [  0,128) gate accumulator of the current head pass  (pg)
-//     [128,256) up accumulator of the current head pass    (pu)
-//     [256,384) g of pass 0, converted in place to alpha = silu'(g) u
-//     [384,512) u of pass 0, converted in place to beta  = silu(g)
+// TMEM (512 columns x 128 lanes = tokens, fp32): two accumulator buffers of
+// 256 columns used by passes alternately, so the epilogue of one pass
+// overlaps the MMAs of the next.
 //
-// Warp roles (320 threads): warp 0 issues TMA loads, warp 1 allocates TMEM
-// and issues the MMAs (one thread), warps 2..9 are the epilogue (two warps
-// per TMEM lane quadrant, each taking 64 of the 128 token columns).
+// Epilogue.  Thread = one token (its TMEM lane); two warps per lane quadrant
+// split the 128 neurons into halves of 64.  Pass 0 leaves alpha = silu'(g) u
+// and beta = silu(g) of the thread's 64 (token, neuron) pairs in registers for
+// the whole unit.  A head pass forms Delta^2 for the same pairs and sums it
+// over tokens: a shuffle butterfly within the warp (32 tokens), then the four
+// quadrant warps' sums are added in shared memory in a fixed order.  The
+// T x G x N intermediate never leaves the SM; each unit writes its G x 128
+// partial sums to its own workspace slot and a second kernel adds them into A
+// in a fixed order, so the result is deterministic.
 //
-// Determinism: every unit writes its per-(half, head, neuron) partial sums to
-// its own workspace slot; a second kernel adds them into A in a fixed order.
+// Warp roles (384 threads, 3 warpgroups): warp 0 issues TMA loads, warp 1
+// allocates TMEM and issues the MMAs (one thread), warps 2-3 idle; warpgroup
+// 0 gives registers back (setmaxnreg) to warpgroups 1-2, the epilogue.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -41,20 +46,25 @@
 namespace dtp {
 namespace tc {
 
-constexpr int BM = 128;       // neurons per tile (MMA M)
-constexpr int BN = 128;       // tokens per chunk (MMA N)
+constexpr int BT = 128;       // tokens per chunk (MMA M, TMEM lanes)
+constexpr int BNEU = 128;     // neurons per tile (MMA N = 2 * BNEU: gate | up)
 constexpr int BK = 64;        // bf16 elements per 128-byte swizzled row
 constexpr int UK = 16;        // K of one tcgen05.mma kind::f16
 constexpr int STAGES = 4;
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;
 constexpr int kEpiWarps = 8;
-constexpr uint32_t kTileA = BM * BK * 2;   // 16 KB, one weight operand
-constexpr uint32_t kTileB = BN * BK * 2;   // 16 KB, activation operand
-constexpr uint32_t kStageBytes = 2 * kTileA + kTileB;
+constexpr int kEpiWarp0 = 4;  // first epilogue warp
+constexpr uint32_t kRegsSmall = 56;   // warpgroup 0 after setmaxnreg.dec
+constexpr uint32_t kRegsLarge = 224;  // epilogue warpgroups after setmaxnreg.inc
+static_assert(128 * kRegsSmall + 256 * kRegsLarge <= kThreads * 168, "register split exceeds the launch budget");
+constexpr uint32_t kTileAct = BT * BK * 2;     // 16 KB activation operand (A)
+constexpr uint32_t kTileW = BNEU * BK * 2;     // 16 KB, W_gate or W_up half of B
+constexpr uint32_t kStageBytes = kTileAct + 2 * kTileW;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColPg = 0, kColPu = 128, kColAlpha = 256, kColBeta = 384;
-constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + 256;
-constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
+constexpr uint32_t kBufCols = 256;
+constexpr size_t kRedBytes = 2 * 4 * BNEU * sizeof(float);   // [slot][quadrant][neuron]
+constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + kRedBytes + 256;
+constexpr uint32_t kIdesc = idesc_bf16_f32(BT, 2 * BNEU);
 
 struct Params {
     int G;          // KV heads
@@ -62,9 +72,27 @@ struct Params {
     int TC;         // token chunks
     int KB;         // k blocks of 64 over d
     int64_t units;  // NT * TC
-    float* partial; // [units][2][G][128]
+    float* partial; // [units][G][128]
     int* status;    // workspace status word
 };
+
+// Sum over the warp's 32 lanes of 32 per-lane columns: afterwards lane L holds
+// the sum of column L.  Each of the 5 rounds halves the columns a lane keeps.
+__device__ __forceinline__ float butterfly32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int r = 0; r < 5; ++r) {
+        const int o = 16 >> r;
+        const int m = 16 >> r;
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < m; ++i) {
+            const float send = upper ? v[i] : v[i + m];
+            const float keep = upper ? v[i + m] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
+        }
+    }
+    return v[0];
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
 affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_constant__ CUtensorMap tm_wu,
@@ -73,16 +101,16 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* tiles = smem;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes);
-    // bars[0..S) full, bars[S..2S) empty, then acc_full, acc_empty, ab_full, ab_empty
+    float* red = reinterpret_cast<float*>(smem + STAGES * kStageBytes);   // [2][4][128]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes + kRedBytes);
+    // full[S], empty[S], acc_full[2], acc_empty[2], red_full[2], drain
     uint64_t* full_bar = bars;
     uint64_t* empty_bar = bars + STAGES;
     uint64_t* acc_full = bars + 2 * STAGES;
-    uint64_t* acc_empty = acc_full + 1;
-    uint64_t* ab_full = acc_full + 2;
-    uint64_t* ab_empty = acc_full + 3;
-    uint64_t* drain_bar = acc_full + 4;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 5);
+    uint64_t* acc_empty = acc_full + 2;
+    uint64_t* red_full = acc_full + 4;
+    uint64_t* drain_bar = acc_full + 6;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 7);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -93,10 +121,11 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
             mbar_init(smem_u32(&full_bar[s]), 1);
             mbar_init(smem_u32(&empty_bar[s]), 1);
         }
-        mbar_init(smem_u32(acc_full), 1);
-        mbar_init(smem_u32(acc_empty), kEpiWarps);
-        mbar_init(smem_u32(ab_full), 1);
-        mbar_init(smem_u32(ab_empty), kEpiWarps);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_empty[b]), kEpiWarps);
+            mbar_init(smem_u32(&red_full[b]), kEpiWarps);
+        }
         mbar_init(smem_u32(drain_bar), 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -113,11 +142,12 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-
     const int passes = p.G + 1;
-    if (warp == 0) {
-        // ------------------------------------------------------------ producer
-        if (lane == 0) {
+
+    if (warp < kEpiWarp0) {
+        setmaxnreg_dec<kRegsSmall>();
+        if (warp == 0 && lane == 0) {
+            // ---------------------------------------------------------------- producer
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_parity[STAGES];
@@ -133,12 +163,12 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                         const uint32_t fb = smem_u32(&full_bar[stage]);
                         uint8_t* st = tiles + stage * kStageBytes;
                         mbar_arrive_expect_tx(fb, kStageBytes);
-                        tma_load_2d(smem_u32(st), &tm_wg, fb, kb * BK, j * BM);
-                        tma_load_2d(smem_u32(st + kTileA), &tm_wu, fb, kb * BK, j * BM);
                         if (pass == 0)
-                            tma_load_2d(smem_u32(st + 2 * kTileA), &tm_x, fb, kb * BK, c * BN);
+                            tma_load_2d(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
                         else
-                            tma_load_3d(smem_u32(st + 2 * kTileA), &tm_c, fb, kb * BK, c * BN, pass - 1);
+                            tma_load_3d(smem_u32(st), &tm_c, fb, kb * BK, c * BT, pass - 1);
+                        tma_load_2d(smem_u32(st + kTileAct), &tm_wg, fb, kb * BK, j * BNEU);
+                        tma_load_2d(smem_u32(st + kTileAct + kTileW), &tm_wu, fb, kb * BK, j * BNEU);
                         issued[stage] = true;
                         issued_parity[stage] = phase;
                         if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -155,48 +185,36 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                         }
                     }
             }
-        }
-    } else if (warp == 1) {
-        // ---------------------------------------------------------- MMA issuer
-        if (lane == 0) {
+        } else if (warp == 1 && lane == 0) {
+            // -------------------------------------------------------------- MMA issuer
             int stage = 0;
-            uint32_t phase = 0, acc_phase = 0, ab_phase = 0;
+            uint32_t phase = 0;
+            uint32_t pass_count = 0;   // over all units: selects the accumulator buffer
             bool ok = true;
             for (int64_t u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-                for (int pass = 0; ok && pass < passes; ++pass) {
-                    uint32_t d_gate, d_up;
-                    if (pass == 0) {
-                        if (!mbar_wait(smem_u32(ab_empty), ab_phase ^ 1u, abort_flag)) { ok = false; break; }
-                        ab_phase ^= 1u;
-                        d_gate = tmem + kColAlpha;
-                        d_up = tmem + kColBeta;
-                    } else {
-                        if (!mbar_wait(smem_u32(acc_empty), acc_phase ^ 1u, abort_flag)) { ok = false; break; }
-                        acc_phase ^= 1u;
-                        d_gate = tmem + kColPg;
-                        d_up = tmem + kColPu;
-                    }
+                for (int pass = 0; ok && pass < passes; ++pass, ++pass_count) {
+                    const uint32_t buf = pass_count & 1u;
+                    const uint32_t use = (pass_count >> 1) & 1u;
+                    if (!mbar_wait(smem_u32(&acc_empty[buf]), use ^ 1u, abort_flag)) { ok = false; break; }
                     tc_fence_after();
+                    const uint32_t d_acc = tmem + buf * kBufCols;
                     for (int kb = 0; kb < p.KB; ++kb) {
                         if (!mbar_wait(smem_u32(&full_bar[stage]), phase, abort_flag)) { ok = false; break; }
                         tc_fence_after();
                         const uint32_t st = smem_u32(tiles + stage * kStageBytes);
-                        const uint64_t dg = smem_desc_k128(st);
-                        const uint64_t du = smem_desc_k128(st + kTileA);
-                        const uint64_t db = smem_desc_k128(st + 2 * kTileA);
+                        const uint64_t da = smem_desc_k128(st);
+                        const uint64_t dw = smem_desc_k128(st + kTileAct);   // 256 rows: W_gate then W_up
 #pragma unroll
                         for (int kk = 0; kk < BK / UK; ++kk) {
                             // advance 16 elements = 32 bytes inside the swizzle atom
                             const uint64_t off = static_cast<uint64_t>((kk * UK * 2) >> 4);
-                            const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
-                            umma_bf16(d_gate, dg + off, db + off, kIdesc, acc);
-                            umma_bf16(d_up, du + off, db + off, kIdesc, acc);
+                            umma_bf16(d_acc, da + off, dw + off, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
                         }
                         umma_commit(smem_u32(&empty_bar[stage]));
                         if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                     }
                     if (!ok) break;
-                    umma_commit(smem_u32(pass == 0 ? ab_full : acc_full));
+                    umma_commit(smem_u32(&acc_full[buf]));
                 }
             }
             // Every MMA must have completed before TMEM is released.
@@ -206,67 +224,86 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
             }
         }
     } else {
-        // ------------------------------------------------------------ epilogue
-        const int quad = warp & 3;
-        const int half = (warp - 2) >> 2;
-        const int row = quad * 32 + lane;                 // neuron within the tile
+        setmaxnreg_inc<kRegsLarge>();
+        // ------------------------------------------------------------------ epilogue
+        const int quad = warp & 3;                         // TMEM lanes 32*quad .. +31 = tokens
+        const int half = (warp - kEpiWarp0) >> 2;          // neurons [64*half, 64*half + 64)
+        const bool summer = (quad == 0);                   // adds the four quadrants of its half
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-        const uint32_t c0 = static_cast<uint32_t>(half * 64);
-        uint32_t acc_phase = 0, ab_phase = 0;
+        const uint32_t col_g = static_cast<uint32_t>(half * 64);          // gate columns of this half
+        const uint32_t col_u = static_cast<uint32_t>(BNEU + half * 64);   // up columns of this half
+        float alpha[64], beta[64];
+        uint32_t pass_count = 0, head_count = 0;
         bool ok = true;
         for (int64_t u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-            // pass 0: convert (g, u) to (alpha, beta) in place
-            if (!mbar_wait(smem_u32(ab_full), ab_phase, abort_flag)) { ok = false; break; }
-            ab_phase ^= 1u;
-            tc_fence_after();
-#pragma unroll 1
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t col = c0 + 16u * i;
-                float g[16], uu[16];
-                tmem_ld16(lane_base + kColAlpha + col, g);
-                tmem_ld16(lane_base + kColBeta + col, uu);
-                tmem_wait_ld();
-                float a[16], b[16];
-#pragma unroll
-                for (int e = 0; e < 16; ++e) swiglu_alpha_beta(g[e], uu[e], a[e], b[e]);
-                tmem_st16(lane_base + kColAlpha + col, a);
-                tmem_st16(lane_base + kColBeta + col, b);
-            }
-            tmem_wait_st();
-            float* out = p.partial + (u * 2 + half) * static_cast<int64_t>(p.G) * BM;
-            for (int h = 0; h < p.G; ++h) {
-                if (!mbar_wait(smem_u32(acc_full), acc_phase, abort_flag)) { ok = false; break; }
-                acc_phase ^= 1u;
+            float* out = p.partial + u * static_cast<int64_t>(p.G) * BNEU;
+            for (int pass = 0; pass < passes; ++pass, ++pass_count) {
+                const uint32_t buf = pass_count & 1u;
+                const uint32_t use = (pass_count >> 1) & 1u;
+                if (!mbar_wait(smem_u32(&acc_full[buf]), use, abort_flag)) { ok = false; break; }
                 tc_fence_after();
-                float pg[64], pu[64];
+                const uint32_t acc = lane_base + buf * kBufCols;
+                if (pass == 0) {
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    tmem_ld16(lane_base + kColPg + c0 + 16u * i, &pg[16 * i]);
-                    tmem_ld16(lane_base + kColPu + c0 + 16u * i, &pu[16 * i]);
+                    for (int i = 0; i < 4; ++i) {
+                        float vg[16], vu[16];
+                        tmem_ld16(acc + col_g + 16u * i, vg);
+                        tmem_ld16(acc + col_u + 16u * i, vu);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            swiglu_alpha_beta(vg[e], vu[e], alpha[16 * i + e], beta[16 * i + e]);
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+                    continue;
                 }
-                tmem_wait_ld();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(acc_empty));
-                float s = 0.0f;
+                // head pass: column sums of Delta^2 over this warp's 32 tokens
+                const uint32_t slot = head_count & 1u;
+                const uint32_t rphase = (head_count >> 1) & 1u;
+                ++head_count;
+                float* rs = red + slot * 4 * BNEU;
+                float colsum[2];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    float a[16], b[16];
-                    tmem_ld16(lane_base + kColAlpha + c0 + 16u * i, a);
-                    tmem_ld16(lane_base + kColBeta + c0 + 16u * i, b);
+                for (int blk = 0; blk < 2; ++blk) {
+                    float d2[32], vu[32];
+                    tmem_ld16(acc + col_g + 32u * blk, &d2[0]);
+                    tmem_ld16(acc + col_g + 32u * blk + 16u, &d2[16]);
+                    tmem_ld16(acc + col_u + 32u * blk, &vu[0]);
+                    tmem_ld16(acc + col_u + 32u * blk + 16u, &vu[16]);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const float dlt = fmaf(a[e], pg[16 * i + e], b[e] * pu[16 * i + e]);
-                        s = fmaf(dlt, dlt, s);
+                    for (int e = 0; e < 32; ++e) {
+                        const float dlt = fmaf(alpha[32 * blk + e], d2[e], beta[32 * blk + e] * vu[e]);
+                        d2[e] = dlt * dlt;
                     }
+                    colsum[blk] = butterfly32(d2, lane);
                 }
-                out[h * BM + row] = s;
+                if (!summer) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+                }
+                rs[quad * BNEU + half * 64 + lane] = colsum[0];
+                rs[quad * BNEU + half * 64 + 32 + lane] = colsum[1];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&red_full[slot]));
+                if (summer) {
+                    // the four quadrants of this half, in a fixed order
+                    if (!mbar_wait(smem_u32(&red_full[slot]), rphase, abort_flag)) { ok = false; break; }
+                    float* o = out + (pass - 1) * BNEU + half * 64;
+#pragma unroll
+                    for (int b = 0; b < 2; ++b) {
+                        const int n = half * 64 + 32 * b + lane;
+                        o[32 * b + lane] = ((rs[n] + rs[BNEU + n]) + rs[2 * BNEU + n]) + rs[3 * BNEU + n];
+                    }
+                    // only now may the buffer (and, two head passes later, this red slot) be reused
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+                }
             }
-            if (!ok) break;
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(ab_empty));
         }
     }
 
@@ -279,7 +316,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
     if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, static_cast<int>(DTP_ERR_NOT_CONVERGED));
 }
 
-// A[h,k] += sum over token chunks (in order) of both column halves' partials.
+// A[h,k] += sum over token chunks (in order) of the unit partials.
 __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
                                        int NT, int TC) {
     const int64_t total = static_cast<int64_t>(G) * N;
@@ -287,12 +324,10 @@ __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float*
          idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int h = static_cast<int>(idx / N);
         const int k = static_cast<int>(idx % N);
-        const int j = k / BM, r = k % BM;
+        const int j = k / BNEU, r = k % BNEU;
         float sum = 0.0f;
-        for (int c = 0; c < TC; ++c) {
-            const int64_t base = ((static_cast<int64_t>(c) * NT + j) * 2) * G * BM + static_cast<int64_t>(h) * BM + r;
-            sum += partial[base] + partial[base + static_cast<int64_t>(G) * BM];
-        }
+        for (int c = 0; c < TC; ++c)
+            sum += partial[((static_cast<int64_t>(c) * NT + j) * G + h) * BNEU + r];
         A[idx] += sum;
     }
 }
@@ -326,9 +361,9 @@ static bool make_map(CUtensorMap* m, const void* base, int rank, const cuuint64_
 
 size_t workspace_bytes(int64_t T, int d, int G, int N) {
     (void)d;
-    const int64_t NT = (N + BM - 1) / BM;
-    const int64_t TC = (T + BN - 1) / BN;
-    return kWorkspaceHeader + static_cast<size_t>(NT * TC) * 2 * G * BM * sizeof(float);
+    const int64_t NT = (N + BNEU - 1) / BNEU;
+    const int64_t TC = (T + BT - 1) / BT;
+    return kWorkspaceHeader + static_cast<size_t>(NT * TC) * G * BNEU * sizeof(float);
 }
 
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
@@ -340,14 +375,14 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
     cuuint64_t dc[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(G)};
     cuuint64_t s2[1] = {row_stride};
     cuuint64_t s3[2] = {row_stride, row_stride * static_cast<cuuint64_t>(T)};
-    if (!make_map(&m_wg, Wg, 2, dw, s2, BM) || !make_map(&m_wu, Wu, 2, dw, s2, BM) ||
-        !make_map(&m_x, X, 2, dx, s2, BN) || !make_map(&m_c, C, 3, dc, s3, BN))
+    if (!make_map(&m_wg, Wg, 2, dw, s2, BNEU) || !make_map(&m_wu, Wu, 2, dw, s2, BNEU) ||
+        !make_map(&m_x, X, 2, dx, s2, BT) || !make_map(&m_c, C, 3, dc, s3, BT))
         return DTP_ERR_CUDA;
 
     Params p;
     p.G = G;
-    p.NT = (N + BM - 1) / BM;
-    p.TC = static_cast<int>((T + BN - 1) / BN);
+    p.NT = (N + BNEU - 1) / BNEU;
+    p.TC = static_cast<int>((T + BT - 1) / BT);
     p.KB = (d + BK - 1) / BK;
     p.units = static_cast<int64_t>(p.NT) * p.TC;
     p.status = reinterpret_cast<int*>(workspace);

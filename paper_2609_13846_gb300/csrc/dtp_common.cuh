@@ -214,6 +214,16 @@ __device__ __forceinline__ void tmem_wait_st() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+// Warpgroup register reallocation (all 128 threads of the warpgroup execute it).
+template <uint32_t kRegs>
+__device__ __forceinline__ void setmaxnreg_inc() {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegs));
+}
+template <uint32_t kRegs>
+__device__ __forceinline__ void setmaxnreg_dec() {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegs));
+}
+
 // SwiGLU operating point of one (neuron, token) pair from its gate and up
 // pre-activations: alpha = silu'(g) u, beta = silu(g) (Sec. 3, equation for
 // Delta).  silu'(g) = s (1 + g (1 - s)) with s the logistic sigmoid.
