@@ -135,8 +135,9 @@ int dtp_affinity_accumulate_noalloc(const void* X, const void* C, const void* W_
 
 /*
  * Synchronises `stream`, then reads the status word that kernels of the last
- * call using `workspace` leave in it: DTP_OK, or DTP_ERR_NOT_CONVERGED if a
- * bounded device-side wait gave up.  workspace_bytes as passed to that call.
+ * call using `workspace` leave in it: DTP_OK, DTP_ERR_NOT_CONVERGED if a
+ * bounded device-side wait or loop gave up, or DTP_ERR_ARG if the layout
+ * search found an invalid entry of A.  workspace_bytes as passed to that call.
  */
 int dtp_workspace_status(const void* workspace, size_t workspace_bytes, void* stream);
 
@@ -177,8 +178,10 @@ int dtp_search_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes)
  *   iters_done  int32 out (device): iterations run (1..iters)
  * Requirements: 2 <= D <= 8, D | H_kv, D | N, H_kv <= 16, N <= 262144,
  * H_kv * N <= 4194304, iters >= 1, the partition count <= 2^26.
- * SYNCHRONOUS: returns after the result is on the device and its status has
- * been read; DTP_ERR_ARG also reports a negative or non-finite entry of A.
+ * Asynchronous on `stream`.  A negative or non-finite entry of A
+ * (DTP_ERR_ARG) or a bounded device loop that hit its limit
+ * (DTP_ERR_NOT_CONVERGED) is reported through the workspace status word,
+ * read with dtp_workspace_status; that layer's outputs are then not written.
  */
 int dtp_search_layout(const float* A, int H_kv, int N, int D, int iters,
                       int32_t* head_part, int32_t* neuron_dev, int64_t* score_q, double* score,
@@ -188,8 +191,9 @@ int dtp_search_layout(const float* A, int H_kv, int N, int D, int iters,
  * dtp_search_layout on `layers` independent layers at once (the up-edge
  * objective decouples across layers); layer i reads A + i*H_kv*N and writes
  * head_part + i*H_kv, neuron_dev + i*N, score_q[i], score[i], iters_done[i].
- * One thread block per layer.  SYNCHRONOUS; returns the first failing
- * layer's status.
+ * One thread block per layer.  Asynchronous; the workspace status word holds
+ * the most severe device-side status over the layers (DTP_ERR_NOT_CONVERGED
+ * before DTP_ERR_ARG before DTP_OK).
  */
 int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D, int iters,
                               int32_t* head_part, int32_t* neuron_dev, int64_t* score_q,

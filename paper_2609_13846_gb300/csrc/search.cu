@@ -45,7 +45,7 @@ constexpr int kFixedBits = 40;
 constexpr int kIdxBits = 18;                       // N <= 2^18
 constexpr int64_t kValBias = int64_t(1) << 45;     // |gain| < 2^44 (H_kv <= 16): fits the 46-bit field
 constexpr int64_t kNegInf = INT64_MIN / 4;
-constexpr size_t kSmemBudget = 200 * 1024;         // dynamic smem for M and nu
+constexpr size_t kSmemBudget = 220 * 1024;         // dynamic smem for M, nu and (if it fits) A
 
 struct Shared {
     uint64_t w[DMAX][DMAX];        // exchange-graph keys (0 = no neuron on the source device)
@@ -67,6 +67,8 @@ struct Shared {
 };
 
 // ---------------------------------------------------------------- helpers --
+
+__device__ __forceinline__ size_t align_up_dev(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // floor(a * 2^(40-e)) for a finite a >= 0, by shifting the fp32 significand.
 __device__ __forceinline__ int64_t quantize(float a, int e) {
@@ -202,7 +204,7 @@ __device__ uint64_t block_select_desc(int n, long long r, KeyFn key, Shared& sh)
 }
 
 struct Layer {
-    const float* A;
+    const float* A;   // the layer's affinities: a shared-memory copy when it fits, else global
     int G, N, D, cap, e;
     int64_t* M;   // [N][D]
     int32_t* nu;  // [N]
@@ -210,11 +212,16 @@ struct Layer {
 
 __device__ void build_gain(const Layer& L, Shared& sh) {
     for (int k = threadIdx.x; k < L.N; k += kThreads) {
+        float a[GMAX];
+#pragma unroll
+        for (int g = 0; g < GMAX; ++g) a[g] = g < L.G ? L.A[static_cast<int64_t>(g) * L.N + k] : 0.0f;
         int64_t m[DMAX];
 #pragma unroll
         for (int l = 0; l < DMAX; ++l) m[l] = 0;
-        for (int g = 0; g < L.G; ++g) {
-            const int64_t q = quantize(L.A[static_cast<int64_t>(g) * L.N + k], L.e);
+#pragma unroll
+        for (int g = 0; g < GMAX; ++g) {
+            if (g >= L.G) break;
+            const int64_t q = quantize(a[g], L.e);
             const int hg = sh.h[g];
 #pragma unroll
             for (int l = 0; l < DMAX; ++l)
@@ -439,25 +446,26 @@ __device__ void neuron_step_general(const Layer& L, Shared& sh) {
 
 // --------------------------------------------------------------- head step --
 
-__device__ void unrank_partition(int64_t idx, int G, int D, int* h) {
+// The idx-th labelled balanced partition in lexicographic order of
+// (h(0), h(1), ...).  With W the number of completions of the current prefix,
+// choosing label l at a position with R groups left leaves W * cnt[l] / R
+// completions (an exact multinomial); all counts stay below 2^30.
+__device__ void unrank_partition(uint32_t idx, uint32_t n_parts, int G, int D, int* h) {
     int cnt[DMAX];
     for (int l = 0; l < D; ++l) cnt[l] = G / D;
-    uint64_t fact[GMAX + 1];
-    fact[0] = 1;
-    for (int i = 1; i <= G; ++i) fact[i] = fact[i - 1] * static_cast<uint64_t>(i);
+    uint32_t W = n_parts;
     for (int g = 0; g < G; ++g) {
-        const int rem = G - g - 1;
+        const uint32_t R = static_cast<uint32_t>(G - g);
         for (int l = 0; l < D; ++l) {
             if (cnt[l] == 0) continue;
-            cnt[l] -= 1;
-            uint64_t ways = fact[rem];
-            for (int m = 0; m < D; ++m) ways /= fact[cnt[m]];
-            if (static_cast<uint64_t>(idx) < ways) {
+            const uint32_t w = W * static_cast<uint32_t>(cnt[l]) / R;
+            if (idx < w) {
                 h[g] = l;
+                W = w;
+                cnt[l] -= 1;
                 break;
             }
-            idx -= static_cast<int64_t>(ways);
-            cnt[l] += 1;
+            idx -= w;
         }
     }
 }
@@ -473,16 +481,28 @@ __device__ bool next_partition(int* h, int G) {
     return true;
 }
 
-__device__ void head_step(const Layer& L, Shared& sh, int64_t n_parts) {
+// (score, index) with the larger score, then the smaller index.
+__device__ __forceinline__ void better(int64_t& s, int& i, int64_t s2, int i2) {
+    if (s2 > s || (s2 == s && i2 < i)) s = s2, i = i2;
+}
+
+__device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
     const int G = L.G, D = L.D;
     if (threadIdx.x < GMAX * DMAX) sh.B[threadIdx.x] = 0;
     __syncthreads();
-    for (int g = 0; g < G; ++g) {
+    // B[g,l]: whole warps per head, each thread a strided slice of the neurons
+    const int warps_per_head = kWarps / G;                 // G <= 16, so >= 2
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = warp / warps_per_head;
+    if (g < G) {
+        const int tph = warps_per_head * 32;
+        const int sub = (warp % warps_per_head) * 32 + lane;
         int64_t acc[DMAX];
 #pragma unroll
         for (int l = 0; l < DMAX; ++l) acc[l] = 0;
-        for (int k = threadIdx.x; k < L.N; k += kThreads) {
-            const int64_t q = quantize(L.A[static_cast<int64_t>(g) * L.N + k], L.e);
+        const float* a = L.A + static_cast<int64_t>(g) * L.N;
+        for (int k = sub; k < L.N; k += tph) {
+            const int64_t q = quantize(a[k], L.e);
             const int l0 = L.nu[k];
 #pragma unroll
             for (int l = 0; l < DMAX; ++l)
@@ -491,31 +511,48 @@ __device__ void head_step(const Layer& L, Shared& sh, int64_t n_parts) {
 #pragma unroll
         for (int l = 0; l < DMAX; ++l)
             if (l < D) {
-                const int64_t s = warp_sum_i64(acc[l]);
-                if ((threadIdx.x & 31) == 0 && s)
-                    atomicAdd(reinterpret_cast<unsigned long long*>(&sh.B[g * D + l]), static_cast<unsigned long long>(s));
+                const int64_t v = warp_sum_i64(acc[l]);
+                if (lane == 0 && v)
+                    atomicAdd(reinterpret_cast<unsigned long long*>(&sh.B[g * D + l]), static_cast<unsigned long long>(v));
             }
     }
     __syncthreads();
-    const int64_t lo = n_parts * threadIdx.x / kThreads;
-    const int64_t hi = n_parts * (threadIdx.x + 1) / kThreads;
+    // score every labelled partition; each thread a contiguous range in lexicographic order
+    const uint32_t lo = static_cast<uint32_t>((static_cast<uint64_t>(n_parts) * threadIdx.x) / kThreads);
+    const uint32_t hi = static_cast<uint32_t>((static_cast<uint64_t>(n_parts) * (threadIdx.x + 1)) / kThreads);
     int64_t best = kNegInf;
-    int64_t best_idx = n_parts;
+    int best_idx = 0x7FFFFFFF;
     if (lo < hi) {
         int hh[GMAX];
-        unrank_partition(lo, G, D, hh);
-        for (int64_t idx = lo; idx < hi; ++idx) {
+        unrank_partition(lo, n_parts, G, D, hh);
+        for (uint32_t idx = lo; idx < hi; ++idx) {
             int64_t s = 0;
-            for (int g = 0; g < G; ++g) s += sh.B[g * D + hh[g]];
-            if (s > best) best = s, best_idx = idx;
+            for (int gg = 0; gg < G; ++gg) s += sh.B[gg * D + hh[gg]];
+            if (s > best) best = s, best_idx = static_cast<int>(idx);
             if (idx + 1 < hi) next_partition(hh, G);
         }
     }
-    const int64_t bmax = block_max_i64(best, sh);
-    const int bidx = block_min_int(best == bmax ? static_cast<int>(best_idx) : 0x7FFFFFFF, sh);
-    if (threadIdx.x == 0) {
-        unrank_partition(bidx, G, D, sh.h);
-        sh.J = bmax;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const int64_t s2 = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+        const int i2 = __shfl_xor_sync(0xFFFFFFFFu, best_idx, o);
+        better(best, best_idx, s2, i2);
+    }
+    if (lane == 0) sh.red_i64[warp] = best, sh.red_int[warp] = best_idx;
+    __syncthreads();
+    if (warp == 0) {
+        int64_t b = sh.red_i64[lane];
+        int bi = sh.red_int[lane];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const int64_t s2 = __shfl_xor_sync(0xFFFFFFFFu, b, o);
+            const int i2 = __shfl_xor_sync(0xFFFFFFFFu, bi, o);
+            better(b, bi, s2, i2);
+        }
+        if (lane == 0) {
+            unrank_partition(static_cast<uint32_t>(bi), n_parts, G, D, sh.h);
+            sh.J = b;
+        }
     }
     __syncthreads();
 }
@@ -526,19 +563,28 @@ __global__ void __launch_bounds__(kThreads, 1)
 search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, int64_t n_parts,
               int32_t* __restrict__ head_out, int32_t* __restrict__ nu_out, int64_t* __restrict__ score_q_out,
               double* __restrict__ score_out, int32_t* __restrict__ iters_out, int* __restrict__ status_out,
-              uint8_t* __restrict__ gbuf, size_t per_layer, int use_smem) {
+              int* __restrict__ ws_status, uint8_t* __restrict__ gbuf, size_t per_layer, int use_smem) {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ Shared sh;
     const int layer = blockIdx.x;
     uint8_t* buf = use_smem ? dsm : gbuf + static_cast<size_t>(layer) * per_layer;
+    const float* A_glob = A_all + static_cast<int64_t>(layer) * G * N;
     Layer L;
-    L.A = A_all + static_cast<int64_t>(layer) * G * N;
+    L.A = A_glob;
     L.G = G;
     L.N = N;
     L.D = D;
     L.cap = N / D;
     L.M = reinterpret_cast<int64_t*>(buf);
     L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * D * sizeof(int64_t));
+    if (use_smem == 2) {
+        // A fits beside M and nu: copy it once; every pass then reads shared memory
+        float* As = reinterpret_cast<float*>(buf + align_up_dev(static_cast<size_t>(N) * D * sizeof(int64_t) +
+                                                                static_cast<size_t>(N) * sizeof(int32_t), 16));
+        for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) As[i] = A_glob[i];
+        __syncthreads();
+        L.A = As;
+    }
 
     if (threadIdx.x == 0) {
         sh.status = DTP_OK;
@@ -555,7 +601,10 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     bad = __syncthreads_or(bad);
     const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
     if (bad) {
-        if (threadIdx.x == 0) status_out[layer] = DTP_ERR_ARG;
+        if (threadIdx.x == 0) {
+            status_out[layer] = DTP_ERR_ARG;
+            atomicMin(ws_status, static_cast<int>(DTP_ERR_ARG));
+        }
         return;
     }
     const float amax = __uint_as_float(static_cast<uint32_t>(amax_all));
@@ -575,7 +624,7 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
         if (D == 2) neuron_step_d2(L, sh);
         else neuron_step_general(L, sh);
         if (sh.status != DTP_OK) break;
-        head_step(L, sh, n_parts);
+        head_step(L, sh, static_cast<uint32_t>(n_parts));
         done = it + 1;
         const bool stop = sh.J <= sh.Jprev;
         __syncthreads();
@@ -585,7 +634,10 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     }
     __syncthreads();
     if (sh.status != DTP_OK) {
-        if (threadIdx.x == 0) status_out[layer] = sh.status;
+        if (threadIdx.x == 0) {
+            status_out[layer] = sh.status;
+            atomicMin(ws_status, sh.status);
+        }
         return;
     }
     for (int k = threadIdx.x; k < N; k += kThreads) nu_out[static_cast<int64_t>(layer) * N + k] = L.nu[k];
@@ -616,6 +668,12 @@ static size_t per_layer_bytes(int N, int D) {
 
 static bool fits_smem(int N, int D) { return per_layer_bytes(N, D) <= kSmemBudget; }
 
+// bytes of M, nu and a copy of A [G,N] fp32 (the layout the kernel uses in mode 2)
+static size_t with_a_bytes(int G, int N, int D) {
+    return align_up(static_cast<size_t>(N) * D * sizeof(int64_t) + static_cast<size_t>(N) * sizeof(int32_t), 16) +
+           static_cast<size_t>(G) * N * sizeof(float);
+}
+
 size_t workspace_bytes(int layers, int G, int N, int D) {
     (void)G;
     size_t b = kWorkspaceHeader + align_up(static_cast<size_t>(layers) * sizeof(int), 256);
@@ -626,32 +684,21 @@ size_t workspace_bytes(int layers, int G, int N, int D) {
 int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* head, int32_t* nu, int64_t* score_q,
            double* score, int32_t* iters_done, void* workspace, cudaStream_t stream) {
     uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+    int* ws_status = reinterpret_cast<int*>(ws);
     int* status = reinterpret_cast<int*>(ws + kWorkspaceHeader);
     uint8_t* gbuf = ws + kWorkspaceHeader + align_up(static_cast<size_t>(layers) * sizeof(int), 256);
     const bool smem = fits_smem(N, D);
-    const size_t dyn = smem ? per_layer_bytes(N, D) : 0;
+    const int mode = !smem ? 0 : (with_a_bytes(G, N, D) <= kSmemBudget ? 2 : 1);
+    const size_t dyn = mode == 2 ? with_a_bytes(G, N, D) : (mode == 1 ? per_layer_bytes(N, D) : 0);
     DTP_CUDA_TRY(cudaFuncSetAttribute(search_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       static_cast<int>(kSmemBudget)));
-    // sentinel 0xFEFEFEFE: a layer whose kernel never reported reads as a CUDA failure
-    DTP_CUDA_TRY(cudaMemsetAsync(status, 0xFE, static_cast<size_t>(layers) * sizeof(int), stream));
+    // the header status word starts at DTP_OK; every block writes its layer's word
+    DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
     search_kernel<<<layers, kThreads, dyn, stream>>>(A, G, N, D, iters, partition_count(G, D), head, nu, score_q,
-                                                      score, iters_done, status, gbuf, per_layer_bytes(N, D),
-                                                      smem ? 1 : 0);
+                                                      score, iters_done, status, ws_status, gbuf,
+                                                      per_layer_bytes(N, D), mode);
     DTP_CUDA_TRY(cudaGetLastError());
-    int* host = static_cast<int*>(malloc(static_cast<size_t>(layers) * sizeof(int)));
-    if (!host) return DTP_ERR_CUDA;
-    cudaError_t err = cudaMemcpyAsync(host, status, static_cast<size_t>(layers) * sizeof(int),
-                                      cudaMemcpyDeviceToHost, stream);
-    if (err == cudaSuccess) err = cudaStreamSynchronize(stream);
-    int rc = DTP_OK;
-    if (err != cudaSuccess) rc = DTP_ERR_CUDA;
-    for (int i = 0; rc == DTP_OK && i < layers; ++i) {
-        const int st = host[i];
-        if (st == DTP_OK) continue;
-        rc = (st == DTP_ERR_ARG || st == DTP_ERR_NOT_CONVERGED) ? st : DTP_ERR_CUDA;
-    }
-    free(host);
-    return rc;
+    return DTP_OK;
 }
 
 }  // namespace search

@@ -186,11 +186,13 @@ def search_workspace_size(layers: int, H_kv: int, N: int, D: int) -> int:
 
 
 def search_layout_batched(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor | None = None,
-                          stream=None) -> dict:
+                          stream=None, check: bool = True) -> dict:
     """Coordinate ascent on each layer of A [L, H_kv, N] (Sec. 3 'Optimiser').
 
     Returns dict of device tensors: h [L,H_kv] int32, nu [L,N] int32,
-    score_q [L] int64, score [L] float64, iters_done [L] int32.  Synchronous.
+    score_q [L] int64, score [L] float64, iters_done [L] int32.  The call is
+    asynchronous; with ``check`` (default) it synchronises and raises
+    DTPError if the device reported a bad entry of A or a loop limit.
     """
     if A.dim() == 2:
         A = A.unsqueeze(0)
@@ -209,10 +211,13 @@ def search_layout_batched(A: torch.Tensor, D: int, iters: int, workspace: torch.
                                          _ptr(out["score_q"]), _ptr(out["score"]), _ptr(out["iters_done"]),
                                          _ptr(workspace), workspace.numel(), _stream(stream))
     _check("dtp_search_layout_batched", st)
+    if check:
+        _check("dtp_search_layout_batched (device status)", workspace_status(workspace, stream))
     return out
 
 
-def search_layout(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor | None = None, stream=None) -> dict:
+def search_layout(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor | None = None, stream=None,
+                  check: bool = True) -> dict:
     """Coordinate ascent on one layer's A [H_kv, N]; tensors as in search_layout_batched, unbatched."""
-    r = search_layout_batched(A.unsqueeze(0) if A.dim() == 2 else A, D, iters, workspace, stream)
+    r = search_layout_batched(A.unsqueeze(0) if A.dim() == 2 else A, D, iters, workspace, stream, check)
     return {k: v[0] for k, v in r.items()}

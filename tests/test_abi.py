@@ -55,7 +55,7 @@ def test_version_and_status_strings(lib):
 def test_workspace_size_queries(lib):
     from paper_2609_13846_gb300 import dtp
     n = dtp.affinity_workspace_size(16384, 1024, 8, 3072, dtp.DTP_BF16)
-    assert n >= 256 + 128 * 24 * 2 * 8 * 128 * 4
+    assert n >= 256 + 128 * 24 * 8 * 128 * 4  # one G x 128 partial per (token chunk, neuron tile)
     assert dtp.affinity_workspace_size(256, 64, 2, 128, dtp.DTP_F32) > 256
     assert dtp.search_workspace_size(28, 8, 3072, 4) >= 256
     # a layer that does not fit in shared memory gets a global buffer
