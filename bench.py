@@ -204,7 +204,7 @@ def main():
         run_reference(args, w)
         return
 
-    from paper_2609_13846_gb300 import dtp
+    from paper_2609_13846_gb300 import dtp, shard
 
     world, rank, local = dist_env()
     torch.cuda.set_device(local)
@@ -214,8 +214,9 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
     peaks = load_peaks()
 
-    # inputs resident in HBM; each rank owns one layer
-    L = synth.make_layer(w.d, w.G, w.N, w.T, w.seed + rank, dtype=w.dtype, outliers=w.outliers, device=dev)
+    # inputs resident in HBM; each rank owns one layer (world layers in all, one block each)
+    layer = shard.layers_for_rank(world, rank, world)[0]
+    L = synth.make_layer(w.d, w.G, w.N, w.T, w.seed + layer, dtype=w.dtype, outliers=w.outliers, device=dev)
     X, C, Wg, Wu = L["X"], L["C"], L["W_gate"], L["W_up"]
     D, iters = w.D[0], w.iters
     A = torch.zeros((w.G, w.N), dtype=torch.float32, device=dev)
@@ -259,13 +260,8 @@ def main():
         t1.record(stream)
         torch.cuda.synchronize()
     barrier()
-    elapsed_ms = t0.elapsed_time(t1)
+    elapsed_ms = shard.max_over_ranks(t0.elapsed_time(t1), device=dev)
     aff_ms = [a.elapsed_time(b) for a, b in aff_ev]
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
     ms_step = elapsed_ms / args.steps
     value = world * w.T * args.steps / (elapsed_ms / 1e3)
     clocks = clk.summary()
@@ -278,6 +274,31 @@ def main():
     s1.record(stream)
     torch.cuda.synchronize()
     search_ms = s0.elapsed_time(s1) / 5
+
+    # the 28-layer Qwen3-0.6B-shaped model search (up-edge objective, all layers batched), on
+    # affinities from this kernel over a 1024-token slice of each layer (seed 100 + layer)
+    model = synth.WORKLOADS["qwen3_0.6b_model"]
+    A_model = torch.zeros((model.layers, model.G, model.N), dtype=torch.float32, device=dev)
+    for i in range(model.layers):
+        Li = synth.make_workload_layer(model, i, T=1024, device=dev)
+        dtp.affinity_accumulate(Li["X"], Li["C"], Li["W_gate"], Li["W_up"], A=A_model[i])
+        del Li
+    model_search = {"layers": model.layers, "tokens_per_layer_for_A": 1024, "iters": model.iters}
+    for Dm in model.D:
+        wsm = torch.empty(dtp.search_workspace_size(model.layers, model.G, model.N, Dm), dtype=torch.uint8, device=dev)
+        rm = dtp.search_layout_batched(A_model, Dm, model.iters, workspace=wsm)
+        m0, m1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        m0.record(stream)
+        for _ in range(5):
+            rm = dtp.search_layout_batched(A_model, Dm, model.iters, workspace=wsm, check=False)
+        m1.record(stream)
+        torch.cuda.synchronize()
+        if dtp.workspace_status(wsm) != dtp.DTP_OK:
+            raise RuntimeError("model search reported a device-side error")
+        model_search[f"D{Dm}_ms"] = m0.elapsed_time(m1) / 5
+        model_search[f"D{Dm}_mean_score"] = float(rm["score"].mean())
+        model_search[f"D{Dm}_max_iters_done"] = int(rm["iters_done"].max())
+    del A_model
 
     # ---- end to end through the public API, host buffers in pinned memory
     hostL = {k: v.cpu().pin_memory() for k, v in L.items()}
@@ -323,6 +344,7 @@ def main():
                    "layers_per_step": world, "l2": "inputs (302 MB) larger than L2; no flush"},
         "affinity_ms": aff_mean_ms, "affinity_tflops": achieved, "search_ms": search_ms,
         "search_iters_done": int(res["iters_done"]), "layout_score": float(res["score"]),
+        "model_search": model_search,
         "roofline": roofline,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": 3 * args.steps,

@@ -210,51 +210,54 @@ struct Layer {
     int32_t* nu;  // [N]
 };
 
+template <int DT>
 __device__ void build_gain(const Layer& L, Shared& sh) {
     for (int k = threadIdx.x; k < L.N; k += kThreads) {
         float a[GMAX];
 #pragma unroll
         for (int g = 0; g < GMAX; ++g) a[g] = g < L.G ? L.A[static_cast<int64_t>(g) * L.N + k] : 0.0f;
-        int64_t m[DMAX];
+        int64_t m[DT];
 #pragma unroll
-        for (int l = 0; l < DMAX; ++l) m[l] = 0;
+        for (int l = 0; l < DT; ++l) m[l] = 0;
 #pragma unroll
         for (int g = 0; g < GMAX; ++g) {
             if (g >= L.G) break;
             const int64_t q = quantize(a[g], L.e);
             const int hg = sh.h[g];
 #pragma unroll
-            for (int l = 0; l < DMAX; ++l)
+            for (int l = 0; l < DT; ++l)
                 if (l == hg) m[l] += q;
         }
-        for (int l = 0; l < L.D; ++l) L.M[static_cast<int64_t>(k) * L.D + l] = m[l];
+#pragma unroll
+        for (int l = 0; l < DT; ++l) L.M[static_cast<int64_t>(k) * DT + l] = m[l];
     }
     __syncthreads();
 }
 
 // Exchange graph over neurons with index > lo: sh.w[a][b] = packed
 // (max gain of moving such a neuron from a to b, lowest index among ties).
+template <int DT>
 __device__ void exchange_graph(const Layer& L, Shared& sh, int lo) {
     if (threadIdx.x < DMAX * DMAX) sh.w[threadIdx.x / DMAX][threadIdx.x % DMAX] = 0;
     __syncthreads();
-    for (int a = 0; a < L.D; ++a) {
-        uint64_t best[DMAX];
+    for (int a = 0; a < DT; ++a) {
+        uint64_t best[DT];
 #pragma unroll
-        for (int b = 0; b < DMAX; ++b) best[b] = 0;
+        for (int b = 0; b < DT; ++b) best[b] = 0;
         for (int k = threadIdx.x; k < L.N; k += kThreads) {
             if (k <= lo || L.nu[k] != a) continue;
-            const int64_t* mk = L.M + static_cast<int64_t>(k) * L.D;
+            const int64_t* mk = L.M + static_cast<int64_t>(k) * DT;
             const int64_t ma = mk[a];
 #pragma unroll
-            for (int b = 0; b < DMAX; ++b)
-                if (b < L.D && b != a) {
+            for (int b = 0; b < DT; ++b)
+                if (b != a) {
                     const uint64_t key = pack_gain(mk[b] - ma, k);
                     best[b] = key > best[b] ? key : best[b];
                 }
         }
 #pragma unroll
-        for (int b = 0; b < DMAX; ++b)
-            if (b < L.D && b != a) {
+        for (int b = 0; b < DT; ++b)
+            if (b != a) {
                 const uint64_t r = warp_max_u64(best[b]);
                 if ((threadIdx.x & 31) == 0 && r) atomicMax(reinterpret_cast<unsigned long long*>(&sh.w[a][b]), r);
             }
@@ -270,11 +273,13 @@ __device__ void count_devices(const Layer& L, Shared& sh) {
 }
 
 // Best device of neuron k at prices pi (lowest index on ties).
+template <int DT>
 __device__ __forceinline__ int best_device(const Layer& L, const Shared& sh, int k) {
-    const int64_t* mk = L.M + static_cast<int64_t>(k) * L.D;
+    const int64_t* mk = L.M + static_cast<int64_t>(k) * DT;
     int best = 0;
     int64_t bv = mk[0] - sh.pi[0];
-    for (int l = 1; l < L.D; ++l) {
+#pragma unroll
+    for (int l = 1; l < DT; ++l) {
         const int64_t v = mk[l] - sh.pi[l];
         if (v > bv) bv = v, best = l;
     }
@@ -321,13 +326,14 @@ __device__ bool apply_path(const Layer& L, const Shared& sh, const int* pred, in
     return true;
 }
 
+template <int DT>
 __device__ void neuron_step_general(const Layer& L, Shared& sh) {
     const int N = L.N, D = L.D, cap = L.cap;
     // (a) price sweeps
     for (int sweep = 0; sweep < 3; ++sweep) {
         if (threadIdx.x < DMAX) sh.count[threadIdx.x] = 0;
         __syncthreads();
-        for (int k = threadIdx.x; k < N; k += kThreads) atomicAdd(&sh.count[best_device(L, sh, k)], 1);
+        for (int k = threadIdx.x; k < N; k += kThreads) atomicAdd(&sh.count[best_device<DT>(L, sh, k)], 1);
         __syncthreads();
         int excess = 0;
         for (int l = 0; l < D; ++l) excess += sh.count[l] > cap ? sh.count[l] - cap : 0;
@@ -349,7 +355,7 @@ __device__ void neuron_step_general(const Layer& L, Shared& sh) {
         }
     }
     // (b) assignment at the current prices
-    for (int k = threadIdx.x; k < N; k += kThreads) L.nu[k] = best_device(L, sh, k);
+    for (int k = threadIdx.x; k < N; k += kThreads) L.nu[k] = best_device<DT>(L, sh, k);
     __syncthreads();
     count_devices(L, sh);
     // (c) successive shortest paths until balanced
@@ -361,7 +367,7 @@ __device__ void neuron_step_general(const Layer& L, Shared& sh) {
         }
         __syncthreads();
         if (sh.flag == 0) break;
-        exchange_graph(L, sh, -1);
+        exchange_graph<DT>(L, sh, -1);
         if (threadIdx.x == 0) {
             unsigned src = 0;
             for (int l = 0; l < D; ++l)
@@ -393,7 +399,7 @@ __device__ void neuron_step_general(const Layer& L, Shared& sh) {
     // (d) lexicographically smallest optimum
     int kstart = 0;
     for (int round = 0; round < N + 1; ++round) {
-        exchange_graph(L, sh, -1);
+        exchange_graph<DT>(L, sh, -1);
         if (threadIdx.x == 0) {
             for (int a = 0; a < D; ++a)
                 for (int b = 0; b < D; ++b)
@@ -423,7 +429,7 @@ __device__ void neuron_step_general(const Layer& L, Shared& sh) {
         }
         const int kstar = block_min_int(cand, sh);
         if (kstar >= N) break;
-        exchange_graph(L, sh, kstar);
+        exchange_graph<DT>(L, sh, kstar);
         if (threadIdx.x == 0) {
             const int t = L.nu[kstar];
             const int64_t* mk = L.M + static_cast<int64_t>(kstar) * D;
@@ -486,6 +492,7 @@ __device__ __forceinline__ void better(int64_t& s, int& i, int64_t s2, int i2) {
     if (s2 > s || (s2 == s && i2 < i)) s = s2, i = i2;
 }
 
+template <int DT>
 __device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
     const int G = L.G, D = L.D;
     if (threadIdx.x < GMAX * DMAX) sh.B[threadIdx.x] = 0;
@@ -497,24 +504,23 @@ __device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
     if (g < G) {
         const int tph = warps_per_head * 32;
         const int sub = (warp % warps_per_head) * 32 + lane;
-        int64_t acc[DMAX];
+        int64_t acc[DT];
 #pragma unroll
-        for (int l = 0; l < DMAX; ++l) acc[l] = 0;
+        for (int l = 0; l < DT; ++l) acc[l] = 0;
         const float* a = L.A + static_cast<int64_t>(g) * L.N;
         for (int k = sub; k < L.N; k += tph) {
             const int64_t q = quantize(a[k], L.e);
             const int l0 = L.nu[k];
 #pragma unroll
-            for (int l = 0; l < DMAX; ++l)
+            for (int l = 0; l < DT; ++l)
                 if (l == l0) acc[l] += q;
         }
 #pragma unroll
-        for (int l = 0; l < DMAX; ++l)
-            if (l < D) {
-                const int64_t v = warp_sum_i64(acc[l]);
-                if (lane == 0 && v)
-                    atomicAdd(reinterpret_cast<unsigned long long*>(&sh.B[g * D + l]), static_cast<unsigned long long>(v));
-            }
+        for (int l = 0; l < DT; ++l) {
+            const int64_t v = warp_sum_i64(acc[l]);
+            if (lane == 0 && v)
+                atomicAdd(reinterpret_cast<unsigned long long*>(&sh.B[g * D + l]), static_cast<unsigned long long>(v));
+        }
     }
     __syncthreads();
     // score every labelled partition; each thread a contiguous range in lexicographic order
@@ -559,6 +565,7 @@ __device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
 
 // ------------------------------------------------------------------ kernel --
 
+template <int DT>
 __global__ void __launch_bounds__(kThreads, 1)
 search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, int64_t n_parts,
               int32_t* __restrict__ head_out, int32_t* __restrict__ nu_out, int64_t* __restrict__ score_q_out,
@@ -620,11 +627,11 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
 
     int done = 0;
     for (int it = 0; it < iters; ++it) {
-        build_gain(L, sh);
-        if (D == 2) neuron_step_d2(L, sh);
-        else neuron_step_general(L, sh);
+        build_gain<DT>(L, sh);
+        if constexpr (DT == 2) neuron_step_d2(L, sh);
+        else neuron_step_general<DT>(L, sh);
         if (sh.status != DTP_OK) break;
-        head_step(L, sh, static_cast<uint32_t>(n_parts));
+        head_step<DT>(L, sh, static_cast<uint32_t>(n_parts));
         done = it + 1;
         const bool stop = sh.J <= sh.Jprev;
         __syncthreads();
@@ -690,11 +697,16 @@ int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* 
     const bool smem = fits_smem(N, D);
     const int mode = !smem ? 0 : (with_a_bytes(G, N, D) <= kSmemBudget ? 2 : 1);
     const size_t dyn = mode == 2 ? with_a_bytes(G, N, D) : (mode == 1 ? per_layer_bytes(N, D) : 0);
-    DTP_CUDA_TRY(cudaFuncSetAttribute(search_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    void (*kernels[DMAX + 1])(const float*, int, int, int, int, int64_t, int32_t*, int32_t*, int64_t*, double*,
+                              int32_t*, int*, int*, uint8_t*, size_t, int) = {
+        nullptr, nullptr, search_kernel<2>, search_kernel<3>, search_kernel<4>,
+        search_kernel<5>, search_kernel<6>, search_kernel<7>, search_kernel<8>};
+    auto kern = kernels[D];
+    DTP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       static_cast<int>(kSmemBudget)));
     // the header status word starts at DTP_OK; every block writes its layer's word
     DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
-    search_kernel<<<layers, kThreads, dyn, stream>>>(A, G, N, D, iters, partition_count(G, D), head, nu, score_q,
+    kern<<<layers, kThreads, dyn, stream>>>(A, G, N, D, iters, partition_count(G, D), head, nu, score_q,
                                                       score, iters_done, status, ws_status, gbuf,
                                                       per_layer_bytes(N, D), mode);
     DTP_CUDA_TRY(cudaGetLastError());
