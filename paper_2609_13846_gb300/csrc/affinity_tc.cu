@@ -17,7 +17,9 @@
 // unit runs G+1 passes over d: pass 0 multiplies the X chunk, pass 1+h the C_h
 // chunk.  Units are dealt round-robin to a persistent grid in
 // token-chunk-major order, so the CTAs in flight share a handful of token
-// chunks in L2 while all weights stay L2-resident.
+// chunks in L2 while all weights stay L2-resident.  The units left over after
+// the last full round are split by heads over several CTAs (each recomputes
+// the unit's X pass), so the final round keeps most SMs busy.
 //
 // TMEM (512 columns x 128 lanes = tokens, fp32): two accumulator buffers of
 // 256 columns used by passes alternately, so the epilogue of one pass
@@ -67,14 +69,41 @@ constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + kRedBytes + 256;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BT, 2 * BNEU);
 
 struct Params {
-    int G;          // KV heads
-    int NT;         // neuron tiles
-    int TC;         // token chunks
-    int KB;         // k blocks of 64 over d
-    int64_t units;  // NT * TC
-    float* partial; // [units][G][128]
-    int* status;    // workspace status word
+    int G;            // KV heads
+    int NT;           // neuron tiles
+    int TC;           // token chunks
+    int KB;           // k blocks of 64 over d
+    int64_t units;    // NT * TC
+    int full_rounds;  // rounds in which every CTA takes one whole unit
+    int split;        // head groups per left-over unit
+    int tail_items;   // left-over units * split (<= grid)
+    float* partial;   // [units][G][128]
+    int* status;      // workspace status word
 };
+
+// The i-th work item of this CTA: a unit and the head range [h0, h1) it covers.
+struct Item {
+    int64_t unit;
+    int h0, h1;
+};
+
+__device__ __forceinline__ bool get_item(const Params& p, int i, Item& it) {
+    if (i < p.full_rounds) {
+        it.unit = static_cast<int64_t>(i) * gridDim.x + blockIdx.x;
+        it.h0 = 0;
+        it.h1 = p.G;
+        return true;
+    }
+    if (i == p.full_rounds && static_cast<int>(blockIdx.x) < p.tail_items) {
+        const int t = static_cast<int>(blockIdx.x);
+        const int grp = t % p.split;
+        it.unit = static_cast<int64_t>(p.full_rounds) * gridDim.x + t / p.split;
+        it.h0 = p.G * grp / p.split;
+        it.h1 = p.G * (grp + 1) / p.split;
+        return true;
+    }
+    return false;
+}
 
 // Sum over the warp's 32 lanes of 32 per-lane columns: afterwards lane L holds
 // the sum of column L.  Each of the 5 rounds halves the columns a lane keeps.
@@ -142,7 +171,6 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const int passes = p.G + 1;
 
     if (warp < kEpiWarp0) {
         setmaxnreg_dec<kRegsSmall>();
@@ -154,9 +182,11 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
             bool issued[STAGES];
             for (int s = 0; s < STAGES; ++s) issued[s] = false, issued_parity[s] = 0;
             bool ok = true;
-            for (int64_t u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-                const int c = static_cast<int>(u / p.NT);
-                const int j = static_cast<int>(u % p.NT);
+            Item it;
+            for (int i = 0; ok && get_item(p, i, it); ++i) {
+                const int c = static_cast<int>(it.unit / p.NT);
+                const int j = static_cast<int>(it.unit % p.NT);
+                const int passes = 1 + it.h1 - it.h0;
                 for (int pass = 0; ok && pass < passes; ++pass) {
                     for (int kb = 0; kb < p.KB; ++kb) {
                         if (!mbar_wait(smem_u32(&empty_bar[stage]), phase ^ 1u, abort_flag)) { ok = false; break; }
@@ -166,7 +196,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                         if (pass == 0)
                             tma_load_2d(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
                         else
-                            tma_load_3d(smem_u32(st), &tm_c, fb, kb * BK, c * BT, pass - 1);
+                            tma_load_3d(smem_u32(st), &tm_c, fb, kb * BK, c * BT, it.h0 + pass - 1);
                         tma_load_2d(smem_u32(st + kTileAct), &tm_wg, fb, kb * BK, j * BNEU);
                         tma_load_2d(smem_u32(st + kTileAct + kTileW), &tm_wu, fb, kb * BK, j * BNEU);
                         issued[stage] = true;
@@ -191,7 +221,9 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
             uint32_t phase = 0;
             uint32_t pass_count = 0;   // over all units: selects the accumulator buffer
             bool ok = true;
-            for (int64_t u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+            Item it;
+            for (int i = 0; ok && get_item(p, i, it); ++i) {
+                const int passes = 1 + it.h1 - it.h0;
                 for (int pass = 0; ok && pass < passes; ++pass, ++pass_count) {
                     const uint32_t buf = pass_count & 1u;
                     const uint32_t use = (pass_count >> 1) & 1u;
@@ -235,8 +267,10 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
         float alpha[64], beta[64];
         uint32_t pass_count = 0, head_count = 0;
         bool ok = true;
-        for (int64_t u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-            float* out = p.partial + u * static_cast<int64_t>(p.G) * BNEU;
+        Item it;
+        for (int i = 0; ok && get_item(p, i, it); ++i) {
+            float* out = p.partial + (it.unit * p.G + it.h0) * static_cast<int64_t>(BNEU);
+            const int passes = 1 + it.h1 - it.h0;
             for (int pass = 0; pass < passes; ++pass, ++pass_count) {
                 const uint32_t buf = pass_count & 1u;
                 const uint32_t use = (pass_count >> 1) & 1u;
@@ -316,19 +350,30 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
     if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, static_cast<int>(DTP_ERR_NOT_CONVERGED));
 }
 
-// A[h,k] += sum over token chunks (in order) of the unit partials.
+// A[h,k] += sum over token chunks of the unit partials.  Eight threads share
+// one output: thread s sums the chunks c = s, s+8, ..., then the eight sums
+// are added in a fixed order, so the result does not depend on scheduling.
+constexpr int kReduceSplit = 8;
 __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
                                        int NT, int TC) {
     const int64_t total = static_cast<int64_t>(G) * N;
-    for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
-         idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int h = static_cast<int>(idx / N);
-        const int k = static_cast<int>(idx % N);
-        const int j = k / BNEU, r = k % BNEU;
+    const int s = threadIdx.x % kReduceSplit;
+    const int64_t per_block = blockDim.x / kReduceSplit;
+    for (int64_t base = blockIdx.x * per_block; base < total; base += static_cast<int64_t>(gridDim.x) * per_block) {
+        const int64_t idx = base + threadIdx.x / kReduceSplit;
         float sum = 0.0f;
-        for (int c = 0; c < TC; ++c)
-            sum += partial[((static_cast<int64_t>(c) * NT + j) * G + h) * BNEU + r];
-        A[idx] += sum;
+        if (idx < total) {
+            const int h = static_cast<int>(idx / N);
+            const int k = static_cast<int>(idx % N);
+            const int j = k / BNEU, r = k % BNEU;
+            for (int c = s; c < TC; c += kReduceSplit)
+                sum += partial[((static_cast<int64_t>(c) * NT + j) * G + h) * BNEU + r];
+        }
+        // fixed-order tree over the 8 lanes of this output (lanes s^4, s^2, s^1)
+        sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 4);
+        sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 2);
+        sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 1);
+        if (idx < total && s == 0) A[idx] += sum;
     }
 }
 
@@ -394,10 +439,17 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
     DTP_CUDA_TRY(cudaFuncSetAttribute(affinity_fo_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       static_cast<int>(kSmemBytes)));
     const int grid = static_cast<int>(p.units < sms ? p.units : sms);
+    p.full_rounds = static_cast<int>(p.units / grid);
+    const int left = static_cast<int>(p.units - static_cast<int64_t>(p.full_rounds) * grid);
+    p.split = left > 0 ? (grid / left < G ? grid / left : G) : 1;
+    if (p.split < 1) p.split = 1;
+    p.tail_items = left * p.split;
     affinity_fo_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(m_wg, m_wu, m_x, m_c, p);
     DTP_CUDA_TRY(cudaGetLastError());
     const int64_t total = static_cast<int64_t>(G) * N;
-    const int rblocks = static_cast<int>((total + 255) / 256 < 4 * sms ? (total + 255) / 256 : 4 * sms);
+    const int64_t outs_per_block = 256 / kReduceSplit;
+    const int64_t want = (total + outs_per_block - 1) / outs_per_block;
+    const int rblocks = static_cast<int>(want < 8 * sms ? want : 8 * sms);
     affinity_reduce_kernel<<<rblocks, 256, 0, stream>>>(p.partial, A, G, N, p.NT, p.TC);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;

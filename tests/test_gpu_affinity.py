@@ -69,6 +69,16 @@ def test_bf16_parity_ragged(d, G, N, T):
     assert np.all(np.abs(A - ref) <= 2e-2 * np.abs(ref) + 1e-6 * np.abs(ref).max())
 
 
+@pytest.mark.parametrize("d,G,N,T", [
+    (64, 8, 1280, 2048),    # 160 units on up to 152 SMs: the 8 left-over units are split by heads
+    (72, 3, 1300, 1900),    # 165 units, 3 heads: left-over units split into single heads
+])
+def test_bf16_parity_left_over_units_split_by_heads(d, G, N, T):
+    L = synth.make_layer(d, G, N, T, seed=G + N, dtype="bf16", outliers=True)
+    A = _gpu(L).cpu().numpy()
+    assert _rel_fro(A, _oracle(L)) <= BF16_TOL
+
+
 @pytest.mark.parametrize("d,G,N,T", [(328, 3, 300, 333), (64, 2, 65, 70)])
 def test_fp32_parity_ragged(d, G, N, T):
     L = synth.make_layer(d, G, N, T, seed=3, dtype="f32", outliers=True)
