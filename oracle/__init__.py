@@ -72,6 +72,21 @@ def _load():
     lib.oracle_search_layout.restype = ctypes.c_int
     lib.oracle_hungarian_max.argtypes = [_i64p, ctypes.c_int, _i32p]
     lib.oracle_hungarian_max.restype = ctypes.c_int64
+    lib.oracle_down_activation.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
+                                           _f64p]
+    lib.oracle_down_activation.restype = None
+    lib.oracle_down_weight_sqnorm.argtypes = [_f64p, _f64p, _f64p, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                              ctypes.c_int, _f64p]
+    lib.oracle_down_weight_sqnorm.restype = None
+    lib.oracle_down_score.argtypes = [_f64p, _f64p, ctypes.c_int, ctypes.c_int, ctypes.c_int64, _f64p]
+    lib.oracle_down_score.restype = None
+    lib.oracle_normalize_unit_mass.argtypes = [_f32p, ctypes.c_int64, _i64p]
+    lib.oracle_normalize_unit_mass.restype = ctypes.c_int
+    lib.oracle_chain_search.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                        ctypes.c_int, _i32p, _i32p, _i64p, _f64p, _i32p, _i32p]
+    lib.oracle_chain_search.restype = ctypes.c_int
+    lib.oracle_chain_score.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p]
+    lib.oracle_chain_score.restype = ctypes.c_int64
     _lib = lib
     return lib
 
@@ -200,3 +215,81 @@ def hungarian_max(W):
     r2c = np.zeros(n, dtype=np.int32)
     total = _load().oracle_hungarian_max(_p(W, _i64p), n, _p(r2c, _i32p))
     return int(total), r2c
+
+
+# --------------------------------------------------------------- down edge ---
+
+def down_activation(X, W_gate, W_up, rms_next):
+    """act2[k] = sum_t (silu(g_k) u_k)^2 / r'_t^2 (Sec. 3, down edge), fp64."""
+    X = _c(X, np.float64)
+    Wg = _c(W_gate, np.float64)
+    Wu = _c(W_up, np.float64)
+    r = _c(rms_next, np.float64)
+    T, d = X.shape
+    N = Wg.shape[0]
+    assert Wg.shape == (N, d) and Wu.shape == (N, d) and r.shape == (T,)
+    out = np.zeros(N, dtype=np.float64)
+    _load().oracle_down_activation(_p(X, _f64p), _p(Wg, _f64p), _p(Wu, _f64p), _p(r, _f64p), T, d, N,
+                                   _p(out, _f64p))
+    return out
+
+
+def down_weight_sqnorm(Wqkv, gamma_next, W_down):
+    """bn[g,k] = ||W^qkv_g (gamma' * w^d_k)||^2 for Wqkv [G,R,d], gamma' [d], W_down [d,N]."""
+    Wq = _c(Wqkv, np.float64)
+    gm = _c(gamma_next, np.float64)
+    Wd = _c(W_down, np.float64)
+    G, R, d = Wq.shape
+    N = Wd.shape[1]
+    assert gm.shape == (d,) and Wd.shape == (d, N)
+    out = np.zeros((G, N), dtype=np.float64)
+    _load().oracle_down_weight_sqnorm(_p(Wq, _f64p), _p(gm, _f64p), _p(Wd, _f64p), G, R, d, N, _p(out, _f64p))
+    return out
+
+
+def down_score(act2, bn, T_total: int):
+    """S_down[g,k] = act2[k] / T_total * bn[g,k] ([G,N], transpose of the paper's I x G)."""
+    a = _c(act2, np.float64)
+    b = _c(bn, np.float64)
+    G, N = b.shape
+    out = np.zeros((G, N), dtype=np.float64)
+    _load().oracle_down_score(_p(a, _f64p), _p(b, _f64p), G, N, T_total, _p(out, _f64p))
+    return out
+
+
+def normalize_unit_mass(S):
+    """Exact integer unit-mass form of one affinity matrix (units of 2^-39)."""
+    S = _c(S, np.float32)
+    n = np.zeros(S.shape, dtype=np.int64)
+    st = _load().oracle_normalize_unit_mass(_p(S, _f32p), S.size, _p(n, _i64p))
+    if st != 0:
+        raise ValueError(f"oracle_normalize_unit_mass: status {st}")
+    return n
+
+
+def chain_search(S_up, S_down, D: int, iters: int):
+    """Coordinate ascent on the whole-model objective (both edges): dict(h, nu, J_q, J, iters_done, unique)."""
+    Su = _c(S_up, np.float32)
+    L, G, N = Su.shape
+    Sd = _c(S_down if L > 1 else np.zeros((1, G, N)), np.float32)
+    assert Sd.shape[1:] == (G, N) and (L == 1 or Sd.shape[0] == L - 1)
+    h = np.zeros((L, G), dtype=np.int32)
+    nu = np.zeros((L, N), dtype=np.int32)
+    jq = ctypes.c_int64(0)
+    j = ctypes.c_double(0.0)
+    it = ctypes.c_int(0)
+    uq = ctypes.c_int(0)
+    st = _load().oracle_chain_search(_p(Su, _f32p), _p(Sd, _f32p), L, G, N, D, iters, _p(h, _i32p), _p(nu, _i32p),
+                                     ctypes.byref(jq), ctypes.byref(j), ctypes.byref(it), ctypes.byref(uq))
+    if st != 0:
+        raise ValueError(f"oracle_chain_search: status {st}")
+    return dict(h=h, nu=nu, J_q=int(jq.value), J=float(j.value), iters_done=int(it.value), unique=bool(uq.value))
+
+
+def chain_score(S_up, S_down, h, nu) -> int:
+    """J of a layout over all layers (Eq. objective), in units of 2^-39."""
+    Su = _c(S_up, np.float32)
+    L, G, N = Su.shape
+    Sd = _c(S_down if L > 1 else np.zeros((1, G, N)), np.float32)
+    return int(_load().oracle_chain_score(_p(Su, _f32p), _p(Sd, _f32p), L, G, N, _p(_c(h, np.int32), _i32p),
+                                          _p(_c(nu, np.int32), _i32p)))

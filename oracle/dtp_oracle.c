@@ -23,6 +23,14 @@
  *                          contiguous head assignment.
  *   oracle_hungarian_max   textbook Hungarian method (Kuhn 1955), used only
  *                          to cross-check the assignment step.
+ *   oracle_down_*          Sec. 3 "Affinity scores", down edge: the write
+ *                          alpha_k w^d_k of neuron k reaches KV group g of the
+ *                          next layer through its pre-norm as (alpha_k/r') b_gk,
+ *                          b_gk = W^qkv_g (gamma' . w^d_k); S_down = E_t[alpha_k^2
+ *                          / r'^2] ||b_gk||^2.
+ *   oracle_normalize_unit_mass, oracle_chain_search
+ *                          Sec. 3 "Objective" (Eq. objective, both sums) and
+ *                          "Optimiser" over all layers of a model.
  *
  * Nothing here is shared with the CUDA library: no header, table or helper.
  * Only the tests, the smoke check and the benchmark's CPU-baseline leg load
@@ -345,11 +353,9 @@ static int lap_extreme(const int64_t* M, int N, int D, const int* nu_opt, int as
  * successive-shortest-path solver for D = 2 as well (used to cross-check the
  * sort).
  */
-int oracle_neuron_step_ex(const int64_t* q, int G, int N, int D, const int* h, int* nu,
-                          int* unique, int general) {
-    if (D < 2 || D > OR_DMAX || N <= 0 || N % D || G <= 0 || G > OR_GMAX) return OR_ERR_ARG;
-    int64_t* M = (int64_t*)malloc(sizeof(int64_t) * (size_t)N * D);
-    build_gain(q, G, N, D, h, M);
+/* Lexicographically smallest balanced assignment maximising sum_k M[k,nu(k)]
+ * for a given gain matrix M [N][D]. */
+static int neuron_step_from_gain(const int64_t* M, int N, int D, int* nu, int* unique, int general) {
     int status = OR_OK;
     if (D == 2 && !general) {
         lap_sort_d2(M, N, nu, unique);
@@ -365,6 +371,15 @@ int oracle_neuron_step_ex(const int64_t* q, int G, int N, int D, const int* h, i
         free(opt);
         free(hi);
     }
+    return status;
+}
+
+int oracle_neuron_step_ex(const int64_t* q, int G, int N, int D, const int* h, int* nu,
+                          int* unique, int general) {
+    if (D < 2 || D > OR_DMAX || N <= 0 || N % D || G <= 0 || G > OR_GMAX) return OR_ERR_ARG;
+    int64_t* M = (int64_t*)malloc(sizeof(int64_t) * (size_t)N * D);
+    build_gain(q, G, N, D, h, M);
+    int status = neuron_step_from_gain(M, N, D, nu, unique, general);
     free(M);
     return status;
 }
@@ -437,6 +452,16 @@ int64_t oracle_count_partitions(int G, int D) {
  * co-located mass of a partition h is sum_g B[g,h(g)]; h = the best labelled
  * balanced partition, lexicographically smallest among ties.
  */
+/* Best labelled balanced partition for column sums B [G][D] (lexicographically smallest among ties). */
+static void head_step_from_sums(const int64_t* B, int G, int D, int* h, int64_t* score) {
+    part_walk s;
+    memset(&s, 0, sizeof(s));
+    s.G = G; s.D = D; s.cap = G / D; s.B = B;
+    part_rec(&s, 0, 0);
+    memcpy(h, s.best, sizeof(int) * (size_t)G);
+    if (score) *score = s.best_score;
+}
+
 int oracle_head_step(const int64_t* q, int G, int N, int D, const int* nu, int* h, int64_t* score) {
     if (D < 2 || D > OR_DMAX || G <= 0 || G % D || G > OR_GMAX || N <= 0) return OR_ERR_ARG;
     int64_t B[OR_GMAX * OR_DMAX];
@@ -495,6 +520,190 @@ int oracle_search_layout(const float* A, int G, int N, int D, int iters, int* h,
     *iters_done = done;
     if (all_unique) *all_unique = uniq_all;
     return OR_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Down edge (Sec. 3 "Affinity scores")                                      */
+/* ------------------------------------------------------------------------ */
+
+/* act2[k] = sum_t alpha_k(t)^2 / r'_t^2 with alpha_k = silu(g_k) u_k, neuron k's
+ * activation on token t, and r'_t the rms of the residual entering the next
+ * layer's pre-norm.  act2 is overwritten. */
+void oracle_down_activation(const double* X, const double* Wg, const double* Wu, const double* rms_next,
+                            int64_t T, int d, int N, double* act2) {
+    #pragma omp parallel for schedule(dynamic, 1)
+    for (int k = 0; k < N; ++k) {
+        const double* wg = Wg + (int64_t)k * d;
+        const double* wu = Wu + (int64_t)k * d;
+        double acc = 0.0;
+        for (int64_t t = 0; t < T; ++t) {
+            const double* x = X + t * d;
+            double g = dot(x, wg, d);
+            double u = dot(x, wu, d);
+            double alpha = g / (1.0 + exp(-g)) * u;
+            double r = rms_next[t];
+            acc += alpha * alpha / (r * r);
+        }
+        act2[k] = acc;
+    }
+}
+
+/* bn[g,k] = || W^qkv_g (gamma' . w^d_k) ||^2 with W^qkv_g the R rows of the next
+ * layer's q/k/v projections that belong to KV group g (Wqkv [G][R][d]), gamma'
+ * the next pre-norm's gain [d] and w^d_k column k of W_down [d][N]. */
+void oracle_down_weight_sqnorm(const double* Wqkv, const double* gamma, const double* Wdown, int G, int R, int d,
+                               int N, double* bn) {
+    #pragma omp parallel for schedule(dynamic, 1)
+    for (int k = 0; k < N; ++k) {
+        double* v = (double*)malloc(sizeof(double) * (size_t)d);
+        for (int i = 0; i < d; ++i) v[i] = gamma[i] * Wdown[(int64_t)i * N + k];
+        for (int g = 0; g < G; ++g) {
+            double acc = 0.0;
+            for (int r = 0; r < R; ++r) {
+                double b = dot(Wqkv + ((int64_t)g * R + r) * d, v, d);
+                acc += b * b;
+            }
+            bn[(int64_t)g * N + k] = acc;
+        }
+        free(v);
+    }
+}
+
+/* S_down[g,k] = act2[k] / T_total * bn[g,k]: the mean over tokens times ||b_gk||^2.
+ * Stored [G][N], the transpose of the paper's I x G orientation. */
+void oracle_down_score(const double* act2, const double* bn, int G, int N, int64_t T_total, double* S) {
+    for (int g = 0; g < G; ++g)
+        for (int k = 0; k < N; ++k)
+            S[(int64_t)g * N + k] = act2[k] / (double)T_total * bn[(int64_t)g * N + k];
+}
+
+/* ------------------------------------------------------------------------ */
+/* Whole-model objective and optimiser (Sec. 3 "Objective", "Optimiser")     */
+/* ------------------------------------------------------------------------ */
+
+#define OR_NORM_BITS 39
+#define OR_NORM_PRE_BITS 24
+
+/*
+ * Unit-mass normalisation (Sec. 3 "Objective": each matrix is normalised to
+ * unit mass so every edge counts equally), in exact integers:
+ *     q = floor(S * 2^(24-e)),  max(S) < 2^e          (q < 2^24)
+ *     n = floor(q * 2^39 / sum(q))                     (sum(n) <= 2^39)
+ * so n is the matrix's share of its own mass in units of 2^-39.  All-zero S
+ * gives n = 0.  Returns -1 for a negative or non-finite entry.
+ */
+int oracle_normalize_unit_mass(const float* S, int64_t count, int64_t* n) {
+    float smax = 0.0f;
+    for (int64_t i = 0; i < count; ++i) {
+        float a = S[i];
+        if (!(a >= 0.0f) || isinf(a)) return OR_ERR_ARG;
+        if (a > smax) smax = a;
+    }
+    if (smax == 0.0f) {
+        for (int64_t i = 0; i < count; ++i) n[i] = 0;
+        return OR_OK;
+    }
+    int e = 0;
+    frexp((double)smax, &e);
+    uint64_t total = 0;
+    for (int64_t i = 0; i < count; ++i) {
+        n[i] = (int64_t)floor(ldexp((double)S[i], OR_NORM_PRE_BITS - e));
+        total += (uint64_t)n[i];
+    }
+    for (int64_t i = 0; i < count; ++i)
+        n[i] = (int64_t)(((uint64_t)n[i] << OR_NORM_BITS) / total);
+    return OR_OK;
+}
+
+/*
+ * Coordinate ascent on J(h, nu) = sum_i up_i + sum_{i<L-1} down_i over L layers,
+ *   up_i   = sum over (g,k) with h_i(g) == nu_i(k)     of nU_i[g,k]
+ *   down_i = sum over (g,k) with nu_i(k) == h_{i+1}(g) of nD_i[g,k]
+ * (nU, nD the unit-mass forms of S_up [L][G][N] and S_down [L-1][G][N]; S_down
+ * stored group-major, the transpose of the paper's I x G).
+ * One iteration: every layer's neuron step given all h (gain M_kl of Sec. 3),
+ * then every layer's head step given all nu (column sums over nu_i for the up
+ * edge and nu_{i-1} for the down edge).  Given the other block, each step
+ * maximises J exactly, so J never decreases.  Start: contiguous heads in every
+ * layer.  Stop after `iters` or the first iteration without a strict increase.
+ * J_q is J in units of 2^-39; *J = J_q / 2^39.
+ */
+int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, int N, int D, int iters, int* h,
+                        int* nu, int64_t* J_q, double* J, int* iters_done, int* all_unique) {
+    if (L < 1 || D < 2 || D > OR_DMAX || G <= 0 || G % D || G > OR_GMAX || N <= 0 || N % D || iters < 1)
+        return OR_ERR_ARG;
+    const int64_t GN = (int64_t)G * N;
+    int64_t* nU = (int64_t*)malloc(sizeof(int64_t) * (size_t)(L * GN));
+    int64_t* nD = (int64_t*)malloc(sizeof(int64_t) * (size_t)((L > 1 ? L - 1 : 1) * GN));
+    int64_t* M = (int64_t*)malloc(sizeof(int64_t) * (size_t)N * D);
+    int status = OR_OK;
+    for (int i = 0; i < L && status == OR_OK; ++i) status = oracle_normalize_unit_mass(S_up + i * GN, GN, nU + i * GN);
+    for (int i = 0; i + 1 < L && status == OR_OK; ++i)
+        status = oracle_normalize_unit_mass(S_down + i * GN, GN, nD + i * GN);
+    for (int i = 0; i < L; ++i)
+        for (int g = 0; g < G; ++g) h[i * G + g] = (g * D) / G;
+    int64_t prev = -1, total = 0;
+    int done = 0, uniq_all = 1;
+    for (int it = 0; it < iters && status == OR_OK; ++it) {
+        for (int i = 0; i < L && status == OR_OK; ++i) {
+            /* M[k,l] = up gain from h_i + down gain from h_{i+1} */
+            memset(M, 0, sizeof(int64_t) * (size_t)N * D);
+            for (int g = 0; g < G; ++g)
+                for (int k = 0; k < N; ++k) {
+                    M[(int64_t)k * D + h[i * G + g]] += nU[i * GN + (int64_t)g * N + k];
+                    if (i + 1 < L) M[(int64_t)k * D + h[(i + 1) * G + g]] += nD[i * GN + (int64_t)g * N + k];
+                }
+            int uniq = 1;
+            status = neuron_step_from_gain(M, N, D, nu + (int64_t)i * N, &uniq, 0);
+            uniq_all &= uniq;
+        }
+        if (status != OR_OK) break;
+        total = 0;
+        for (int i = 0; i < L; ++i) {
+            /* B[g,l] = up mass of g on device l under nu_i + down mass into g under nu_{i-1} */
+            int64_t B[OR_GMAX * OR_DMAX];
+            memset(B, 0, sizeof(B));
+            for (int g = 0; g < G; ++g)
+                for (int k = 0; k < N; ++k) {
+                    B[g * D + nu[(int64_t)i * N + k]] += nU[i * GN + (int64_t)g * N + k];
+                    if (i > 0) B[g * D + nu[(int64_t)(i - 1) * N + k]] += nD[(i - 1) * GN + (int64_t)g * N + k];
+                }
+            int64_t sc = 0;
+            head_step_from_sums(B, G, D, h + i * G, &sc);
+            total += sc;
+        }
+        done = it + 1;
+        if (total <= prev) break;
+        prev = total;
+    }
+    free(nU); free(nD); free(M);
+    if (status != OR_OK) return status;
+    *J_q = total;
+    *J = ldexp((double)total, -OR_NORM_BITS);
+    *iters_done = done;
+    if (all_unique) *all_unique = uniq_all;
+    return OR_OK;
+}
+
+/* J of a given layout (both sums of Eq. objective), in units of 2^-39. */
+int64_t oracle_chain_score(const float* S_up, const float* S_down, int L, int G, int N, const int* h, const int* nu) {
+    const int64_t GN = (int64_t)G * N;
+    int64_t* n = (int64_t*)malloc(sizeof(int64_t) * (size_t)GN);
+    int64_t J = 0;
+    for (int i = 0; i < L; ++i) {
+        if (oracle_normalize_unit_mass(S_up + i * GN, GN, n) != OR_OK) { J = -1; break; }
+        for (int g = 0; g < G; ++g)
+            for (int k = 0; k < N; ++k)
+                if (h[i * G + g] == nu[(int64_t)i * N + k]) J += n[(int64_t)g * N + k];
+        if (i + 1 < L) {
+            if (oracle_normalize_unit_mass(S_down + i * GN, GN, n) != OR_OK) { J = -1; break; }
+            for (int g = 0; g < G; ++g)
+                for (int k = 0; k < N; ++k)
+                    if (nu[(int64_t)i * N + k] == h[(i + 1) * G + g]) J += n[(int64_t)g * N + k];
+        }
+    }
+    free(n);
+    return J;
 }
 
 /* ------------------------------------------------------------------------ */
