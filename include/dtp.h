@@ -94,6 +94,65 @@ int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, co
                             void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * dtp_affinity_accumulate plus the down-edge activation term of Sec. 3
+ * ("Affinity scores", down edge: neuron k writes alpha_k w^d_k into the
+ * residual, alpha_k = silu(g_k) u_k its activation):
+ *     act2[k] += sum_{t<T} alpha_k(t)^2 / rms_next[t]^2
+ *   rms_next [T] fp32  rms r' of the residual entering the next layer's
+ *                      pre-norm (> 0)
+ *   act2     [N] fp32  accumulated
+ * rms_next and act2 are both NULL (then this is dtp_affinity_accumulate) or
+ * both set.  The workspace is sized by dtp_affinity_workspace_size, which
+ * covers both forms.  A is bitwise the same as without the extra term.
+ */
+int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate, const void* W_up,
+                               const float* rms_next, int64_t T, int d, int H_kv, int N, int dtype,
+                               float* A, float* act2, void* workspace, size_t workspace_bytes,
+                               void* stream);
+
+/*
+ * The ADD score of Sec. 3 before the mean: the squared additive contribution
+ * of KV group h's piece to neuron k's pre-activations, ignoring the operating
+ * point and ||w^d_k||:
+ *     A_add[h,k] += sum_{t<T} (c_{h,t} . w^g_k)^2 + (c_{h,t} . w^u_k)^2
+ * C [H_kv, T, d], W_gate/W_up [N, d] bf16; A_add [H_kv, N] fp32 accumulated.
+ * Same size rules as dtp_affinity_accumulate; workspace from
+ * dtp_affinity_add_workspace_size.  Deterministic.  Asynchronous.
+ */
+int dtp_affinity_add_workspace_size(int64_t T, int d, int H_kv, int N, size_t* bytes);
+int dtp_affinity_add_accumulate(const void* C, const void* W_gate, const void* W_up, int64_t T, int d,
+                                int H_kv, int N, float* A_add, void* workspace,
+                                size_t workspace_bytes, void* stream);
+
+/*
+ * Down-edge weight factor (Sec. 3): bn[g,k] = ||b_gk||^2 with
+ * b_gk = W^qkv_g (gamma' . w^d_k), the column w^d_k of this layer's down
+ * projection seen by KV group g of the next layer through its pre-norm gain.
+ *   Wqkv_next  [H_kv, R, d] bf16: the next layer's q, k and v projection rows of
+ *              each KV group (the group's query heads with its key and value
+ *              head), R rows per group
+ *   gamma_next [d] bf16: the next layer's attention pre-norm gain
+ *   W_down     [d, N] bf16 (nn.Linear [out=d, in=N])
+ *   bn         [H_kv, N] fp32 out (overwritten)
+ * gamma' . w^d_k is rounded to bf16 once before the tensor-core product.
+ * Requirements: d % 8 == 0; dtype DTP_BF16 (others: DTP_ERR_UNSUPPORTED).
+ * Workspace from dtp_down_weight_workspace_size.  Asynchronous.
+ */
+int dtp_down_weight_workspace_size(int H_kv, int R, int d, int N, size_t* bytes);
+int dtp_down_weight_sqnorm(const void* Wqkv_next, const void* gamma_next, const void* W_down,
+                           int H_kv, int R, int d, int N, int dtype, float* bn, void* workspace,
+                           size_t workspace_bytes, void* stream);
+
+/*
+ * The down-edge affinity of Sec. 3: S_down[g,k] = act2[k] / T_total * bn[g,k]
+ * = E_t[alpha_k^2 / r'^2] ||b_gk||^2, how much KV group g of the next layer
+ * depends on neuron k of this layer.  Stored [H_kv, N] (the transpose of the
+ * paper's I x G orientation).  All device fp32.  Asynchronous.
+ */
+int dtp_down_finalize(const float* act2, const float* bn, int H_kv, int N, int64_t T_total,
+                      float* S_down, void* stream);
+
+/*
  * A[h,k] *= wd_sqnorm[k] / T_total, the token mean E_t and the squared norm of
  * neuron k's down-projection column (Sec. 3, S^{up,fo} = E_t[Delta^2] ||w^d_k||^2).
  * wd_sqnorm: device fp32 [N], or NULL for a factor of 1.  T_total >= 1.

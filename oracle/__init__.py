@@ -72,6 +72,9 @@ def _load():
     lib.oracle_search_layout.restype = ctypes.c_int
     lib.oracle_hungarian_max.argtypes = [_i64p, ctypes.c_int, _i32p]
     lib.oracle_hungarian_max.restype = ctypes.c_int64
+    lib.oracle_affinity_add.argtypes = [_f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
+                                        ctypes.c_int, _f64p]
+    lib.oracle_affinity_add.restype = None
     lib.oracle_down_activation.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
                                            _f64p]
     lib.oracle_down_activation.restype = None
@@ -120,6 +123,18 @@ def affinity_fo(X, C, W_gate, W_up) -> np.ndarray:
     A = np.zeros((G, N), dtype=np.float64)
     _load().oracle_affinity_fo(_p(X, _f64p), _p(C, _f64p), _p(Wg, _f64p), _p(Wu, _f64p),
                                T, d, G, N, _p(A, _f64p))
+    return A
+
+
+def affinity_add(C, W_gate, W_up) -> np.ndarray:
+    """ADD score before the mean: sum_t (p_h . w^g_k)^2 + (p_h . w^u_k)^2 (Sec. 3), fp64."""
+    C = _c(C, np.float64)
+    Wg = _c(W_gate, np.float64)
+    Wu = _c(W_up, np.float64)
+    G, T, d = C.shape
+    N = Wg.shape[0]
+    A = np.zeros((G, N), dtype=np.float64)
+    _load().oracle_affinity_add(_p(C, _f64p), _p(Wg, _f64p), _p(Wu, _f64p), T, d, G, N, _p(A, _f64p))
     return A
 
 

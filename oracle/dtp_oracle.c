@@ -110,6 +110,29 @@ void oracle_affinity_fo(const double* X, const double* C, const double* Wg, cons
     }
 }
 
+/* The ADD score of Sec. 3 before the mean: A_add[h,k] = sum_t (p_h . w^g_k)^2 +
+ * (p_h . w^u_k)^2, the squared additive contribution of head h's piece to
+ * neuron k's two pre-activations (no operating point, no ||w^d_k||).
+ * A_add is overwritten. */
+void oracle_affinity_add(const double* C, const double* Wg, const double* Wu, int64_t T, int d, int G, int N,
+                         double* A) {
+    #pragma omp parallel for schedule(dynamic, 1)
+    for (int k = 0; k < N; ++k) {
+        const double* wg = Wg + (int64_t)k * d;
+        const double* wu = Wu + (int64_t)k * d;
+        for (int h = 0; h < G; ++h) {
+            double acc = 0.0;
+            for (int64_t t = 0; t < T; ++t) {
+                const double* p = C + ((int64_t)h * T + t) * d;
+                double pg = dot(p, wg, d);
+                double pu = dot(p, wu, d);
+                acc += pg * pg + pu * pu;
+            }
+            A[(int64_t)h * N + k] = acc;
+        }
+    }
+}
+
 /* A[h,k] *= wd_sqnorm[k] / T_total  (E_t mean and the ||w^d_k||^2 factor);
  * wd_sqnorm == NULL means the factor 1. */
 void oracle_finalize(double* A, int G, int N, int64_t T_total, const double* wd_sqnorm) {

@@ -67,7 +67,8 @@ __device__ __forceinline__ void tile_gemm(const float* __restrict__ act, int64_t
 
 __global__ void __launch_bounds__(kThreads)
 affinity_fo_f32_kernel(const float* __restrict__ X, const float* __restrict__ C, const float* __restrict__ Wg,
-                       const float* __restrict__ Wu, int64_t T, int d, int G, int N, float* __restrict__ partial) {
+                       const float* __restrict__ Wu, int64_t T, int d, int G, int N, float* __restrict__ partial,
+                       const float* __restrict__ rms, float* __restrict__ partial_act) {
     __shared__ float xs[TK][TT + 1];
     __shared__ float gs[TK][TN + 1];
     __shared__ float us[TK][TN + 1];
@@ -88,6 +89,31 @@ affinity_fo_f32_kernel(const float* __restrict__ X, const float* __restrict__ C,
             beta[i][j] = g * s;
             alpha[i][j] = s * (1.0f + g * (1.0f - s)) * u;
         }
+    if (rms) {
+        // down-edge activation term: sum over this tile's tokens of (silu(g) u)^2 / r'^2
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            float s = 0.0f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int64_t t = t0 + ty + 16 * i;
+                if (t < T) {
+                    const float act = beta[i][j] * acc_u[i][j];
+                    const float r = rms[t];
+                    s = fmaf(act * act, 1.0f / (r * r), s);
+                }
+            }
+            red[ty][tx + 16 * j] = s;
+        }
+        __syncthreads();
+        if (threadIdx.x < TN) {
+            float s = 0.0f;
+            for (int r = 0; r < 16; ++r) s += red[r][threadIdx.x];
+            const int n = n0 + threadIdx.x;
+            if (n < N) partial_act[tile * N + n] = s;
+        }
+        __syncthreads();
+    }
     for (int h = 0; h < G; ++h) {
         tile_gemm(C + static_cast<int64_t>(h) * T * d, T, d, Wg, Wu, N, t0, n0, acc_g, acc_u, xs, gs, us);
 #pragma unroll
@@ -112,35 +138,54 @@ affinity_fo_f32_kernel(const float* __restrict__ X, const float* __restrict__ C,
 }
 
 __global__ void f32_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
-                                  int64_t tiles) {
-    const int64_t total = static_cast<int64_t>(G) * N;
+                                  int64_t tiles, const float* __restrict__ partial_act, float* __restrict__ act2) {
+    const int64_t total_a = static_cast<int64_t>(G) * N;
+    const int64_t total = total_a + (act2 ? N : 0);
     for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
          idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         float s = 0.0f;
-        for (int64_t t = 0; t < tiles; ++t) s += partial[t * total + idx];
-        A[idx] += s;
+        if (idx < total_a) {
+            for (int64_t t = 0; t < tiles; ++t) s += partial[t * total_a + idx];
+            A[idx] += s;
+        } else {
+            const int64_t k = idx - total_a;
+            for (int64_t t = 0; t < tiles; ++t) s += partial_act[t * N + k];
+            act2[k] += s;
+        }
     }
 }
 
 size_t workspace_bytes(int64_t T, int d, int G, int N) {
     (void)d;
     const int64_t tiles = (T + TT - 1) / TT;
-    return kWorkspaceHeader + static_cast<size_t>(tiles) * G * N * sizeof(float);
+    return kWorkspaceHeader + static_cast<size_t>(tiles) * (G + 1) * N * sizeof(float);
 }
 
 int launch(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
-           float* A, void* workspace, cudaStream_t stream) {
+           float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2) {
     const int64_t tiles = (T + TT - 1) / TT;
     if (tiles > 65535) return DTP_ERR_UNSUPPORTED;
     float* partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(workspace) + kWorkspaceHeader);
+    float* partial_act = partial + tiles * static_cast<int64_t>(G) * N;
+    const bool want_act = rms && act2;
     dim3 grid((N + TN - 1) / TN, static_cast<unsigned>(tiles));
-    affinity_fo_f32_kernel<<<grid, kThreads, 0, stream>>>(X, C, Wg, Wu, T, d, G, N, partial);
+    affinity_fo_f32_kernel<<<grid, kThreads, 0, stream>>>(X, C, Wg, Wu, T, d, G, N, partial,
+                                                          want_act ? rms : nullptr, partial_act);
     DTP_CUDA_TRY(cudaGetLastError());
-    const int64_t total = static_cast<int64_t>(G) * N;
+    const int64_t total = static_cast<int64_t>(G) * N + (want_act ? N : 0);
     const int blocks = static_cast<int>((total + 255) / 256 < 1024 ? (total + 255) / 256 : 1024);
-    f32_reduce_kernel<<<blocks, 256, 0, stream>>>(partial, A, G, N, tiles);
+    f32_reduce_kernel<<<blocks, 256, 0, stream>>>(partial, A, G, N, tiles, partial_act, want_act ? act2 : nullptr);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
+}
+
+// S_down[g,k] = act2[k] / T_total * bn[g,k]
+__global__ void down_finalize_kernel(const float* __restrict__ act2, const float* __restrict__ bn, int G, int N,
+                                     float inv_t, float* __restrict__ S) {
+    const int64_t total = static_cast<int64_t>(G) * N;
+    for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
+         idx += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        S[idx] = act2[idx % N] * inv_t * bn[idx];
 }
 
 }  // namespace f32
@@ -169,6 +214,16 @@ __global__ void down_sqnorm_kernel(const T* __restrict__ W, int d, int N, float*
         s = fmaf(w, w, s);
     }
     out[k] = s;
+}
+
+int launch_down_finalize(const float* act2, const float* bn, int G, int N, int64_t T_total, float* S,
+                         cudaStream_t stream) {
+    const int64_t total = static_cast<int64_t>(G) * N;
+    const int blocks = static_cast<int>((total + 255) / 256 < 1024 ? (total + 255) / 256 : 1024);
+    f32::down_finalize_kernel<<<blocks, 256, 0, stream>>>(act2, bn, G, N,
+                                                         static_cast<float>(1.0 / static_cast<double>(T_total)), S);
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
 }
 
 int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream) {

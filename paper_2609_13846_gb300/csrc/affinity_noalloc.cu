@@ -29,7 +29,7 @@ namespace dtp {
 namespace tc {
 size_t workspace_bytes(int64_t T, int d, int G, int N);
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
-           void* workspace, cudaStream_t stream);
+           void* workspace, cudaStream_t stream, const float* rms, float* act2);
 }  // namespace tc
 }  // namespace dtp
 
@@ -82,5 +82,5 @@ extern "C" int dtp_affinity_accumulate_noalloc(const void* X, const void* C, con
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // The status word must start at zero; the partial sums are all written before they are read.
     if (cudaMemsetAsync(scratch, 0, dtp::kWorkspaceHeader, s) != cudaSuccess) return DTP_ERR_CUDA;
-    return dtp::tc::launch(X, C, W_gate, W_up, T, d, H_kv, N, A, scratch, s);
+    return dtp::tc::launch(X, C, W_gate, W_up, T, d, H_kv, N, A, scratch, s, nullptr, nullptr);
 }

@@ -35,6 +35,11 @@
 // partial sums to its own workspace slot and a second kernel adds them into A
 // in a fixed order, so the result is deterministic.
 //
+// Down-edge activation term (optional): with the rms r' of the residual that
+// enters the next layer's pre-norm, the X pass also sums (silu(g) u)^2 / r'^2
+// over tokens per neuron -- E_t[alpha_k^2 / r'^2] of the down-edge score before
+// the mean -- with the same butterfly and quadrant reduction.
+//
 // Warp roles (384 threads, 3 warpgroups): warp 0 issues TMA loads, warp 1
 // allocates TMEM and issues the MMAs (one thread), warps 2-3 idle; warpgroup
 // 0 gives registers back (setmaxnreg) to warpgroups 1-2, the epilogue.
@@ -77,7 +82,10 @@ struct Params {
     int full_rounds;  // rounds in which every CTA takes one whole unit
     int split;        // head groups per left-over unit
     int tail_items;   // left-over units * split (<= grid)
+    int64_t T;        // tokens
     float* partial;   // [units][G][128]
+    const float* rms; // [T] rms of the next layer's pre-norm input, or null
+    float* partial_act;  // [units][128] down-edge activation sums (when rms is set)
     int* status;      // workspace status word
 };
 
@@ -267,6 +275,37 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
         float alpha[64], beta[64];
         uint32_t pass_count = 0, head_count = 0;
         bool ok = true;
+        // Adds this warp's two 32-column sums into the four-quadrant sum of its half and, for
+        // the summing warps, writes the 64 results to dst and releases the TMEM buffer.
+        auto reduce_store = [&](const float (&colsum)[2], float* dst, uint32_t buf) -> bool {
+            const uint32_t slot = head_count & 1u;
+            const uint32_t rphase = (head_count >> 1) & 1u;
+            ++head_count;
+            float* rs = red + slot * 4 * BNEU;
+            if (!summer) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+            }
+            rs[quad * BNEU + half * 64 + lane] = colsum[0];
+            rs[quad * BNEU + half * 64 + 32 + lane] = colsum[1];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&red_full[slot]));
+            if (summer) {
+                // the four quadrants of this half, in a fixed order
+                if (!mbar_wait(smem_u32(&red_full[slot]), rphase, abort_flag)) return false;
+#pragma unroll
+                for (int b = 0; b < 2; ++b) {
+                    const int n = half * 64 + 32 * b + lane;
+                    dst[32 * b + lane] = ((rs[n] + rs[BNEU + n]) + rs[2 * BNEU + n]) + rs[3 * BNEU + n];
+                }
+                // only now may the buffer (and, two reductions later, this red slot) be reused
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+            }
+            return true;
+        };
         Item it;
         for (int i = 0; ok && get_item(p, i, it); ++i) {
             float* out = p.partial + (it.unit * p.G + it.h0) * static_cast<int64_t>(BNEU);
@@ -278,26 +317,43 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                 tc_fence_after();
                 const uint32_t acc = lane_base + buf * kBufCols;
                 if (pass == 0) {
+                    // operating point; optionally the down-edge activation sums
+                    const bool want_act = p.rms != nullptr && it.h0 == 0;
+                    float ir2 = 0.0f;
+                    if (want_act) {
+                        const int64_t tok = (it.unit / p.NT) * BT + quad * 32 + lane;
+                        if (tok < p.T) {
+                            const float r = p.rms[tok];
+                            ir2 = 1.0f / (r * r);
+                        }
+                    }
+                    float asum[2];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        float vg[16], vu[16];
-                        tmem_ld16(acc + col_g + 16u * i, vg);
-                        tmem_ld16(acc + col_u + 16u * i, vu);
+                    for (int blk = 0; blk < 2; ++blk) {
+                        float vg[32], vu[32];
+                        tmem_ld16(acc + col_g + 32u * blk, &vg[0]);
+                        tmem_ld16(acc + col_g + 32u * blk + 16u, &vg[16]);
+                        tmem_ld16(acc + col_u + 32u * blk, &vu[0]);
+                        tmem_ld16(acc + col_u + 32u * blk + 16u, &vu[16]);
                         tmem_wait_ld();
 #pragma unroll
-                        for (int e = 0; e < 16; ++e)
-                            swiglu_alpha_beta(vg[e], vu[e], alpha[16 * i + e], beta[16 * i + e]);
+                        for (int e = 0; e < 32; ++e) {
+                            swiglu_alpha_beta(vg[e], vu[e], alpha[32 * blk + e], beta[32 * blk + e]);
+                            const float act = beta[32 * blk + e] * vu[e];   // silu(g) u
+                            vg[e] = act * act * ir2;
+                        }
+                        asum[blk] = want_act ? butterfly32(vg, lane) : 0.0f;
                     }
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+                    if (!want_act) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+                        continue;
+                    }
+                    if (!reduce_store(asum, p.partial_act + it.unit * BNEU + half * 64, buf)) { ok = false; break; }
                     continue;
                 }
                 // head pass: column sums of Delta^2 over this warp's 32 tokens
-                const uint32_t slot = head_count & 1u;
-                const uint32_t rphase = (head_count >> 1) & 1u;
-                ++head_count;
-                float* rs = red + slot * 4 * BNEU;
                 float colsum[2];
 #pragma unroll
                 for (int blk = 0; blk < 2; ++blk) {
@@ -314,29 +370,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                     }
                     colsum[blk] = butterfly32(d2, lane);
                 }
-                if (!summer) {
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
-                }
-                rs[quad * BNEU + half * 64 + lane] = colsum[0];
-                rs[quad * BNEU + half * 64 + 32 + lane] = colsum[1];
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&red_full[slot]));
-                if (summer) {
-                    // the four quadrants of this half, in a fixed order
-                    if (!mbar_wait(smem_u32(&red_full[slot]), rphase, abort_flag)) { ok = false; break; }
-                    float* o = out + (pass - 1) * BNEU + half * 64;
-#pragma unroll
-                    for (int b = 0; b < 2; ++b) {
-                        const int n = half * 64 + 32 * b + lane;
-                        o[32 * b + lane] = ((rs[n] + rs[BNEU + n]) + rs[2 * BNEU + n]) + rs[3 * BNEU + n];
-                    }
-                    // only now may the buffer (and, two head passes later, this red slot) be reused
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
-                }
+                if (!reduce_store(colsum, out + (pass - 1) * BNEU + half * 64, buf)) { ok = false; break; }
             }
         }
     }
@@ -355,25 +389,34 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
 // are added in a fixed order, so the result does not depend on scheduling.
 constexpr int kReduceSplit = 8;
 __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
-                                       int NT, int TC) {
-    const int64_t total = static_cast<int64_t>(G) * N;
+                                       int NT, int TC, const float* __restrict__ partial_act,
+                                       float* __restrict__ act2) {
+    const int64_t total_a = static_cast<int64_t>(G) * N;
+    const int64_t total = total_a + (act2 ? N : 0);
     const int s = threadIdx.x % kReduceSplit;
     const int64_t per_block = blockDim.x / kReduceSplit;
     for (int64_t base = blockIdx.x * per_block; base < total; base += static_cast<int64_t>(gridDim.x) * per_block) {
         const int64_t idx = base + threadIdx.x / kReduceSplit;
         float sum = 0.0f;
-        if (idx < total) {
+        if (idx < total_a) {
             const int h = static_cast<int>(idx / N);
             const int k = static_cast<int>(idx % N);
             const int j = k / BNEU, r = k % BNEU;
             for (int c = s; c < TC; c += kReduceSplit)
                 sum += partial[((static_cast<int64_t>(c) * NT + j) * G + h) * BNEU + r];
+        } else if (idx < total) {
+            const int k = static_cast<int>(idx - total_a);
+            const int j = k / BNEU, r = k % BNEU;
+            for (int c = s; c < TC; c += kReduceSplit) sum += partial_act[(static_cast<int64_t>(c) * NT + j) * BNEU + r];
         }
         // fixed-order tree over the 8 lanes of this output (lanes s^4, s^2, s^1)
         sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 4);
         sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 2);
         sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 1);
-        if (idx < total && s == 0) A[idx] += sum;
+        if (s == 0) {
+            if (idx < total_a) A[idx] += sum;
+            else if (idx < total) act2[idx - total_a] += sum;
+        }
     }
 }
 
@@ -404,15 +447,27 @@ static bool make_map(CUtensorMap* m, const void* base, int rank, const cuuint64_
     return r == CUDA_SUCCESS;
 }
 
-size_t workspace_bytes(int64_t T, int d, int G, int N) {
-    (void)d;
+static size_t partial_bytes(int64_t T, int G, int N) {
     const int64_t NT = (N + BNEU - 1) / BNEU;
     const int64_t TC = (T + BT - 1) / BT;
-    return kWorkspaceHeader + static_cast<size_t>(NT * TC) * G * BNEU * sizeof(float);
+    return static_cast<size_t>(NT * TC) * G * BNEU * sizeof(float);
+}
+
+// bytes of the header and the per-unit A partials (the down-edge activation
+// partials, one more 128-float row per unit, come after them when requested)
+size_t workspace_bytes(int64_t T, int d, int G, int N) {
+    (void)d;
+    return kWorkspaceHeader + partial_bytes(T, G, N);
+}
+
+size_t workspace_bytes_with_act(int64_t T, int d, int G, int N) {
+    const int64_t NT = (N + BNEU - 1) / BNEU;
+    const int64_t TC = (T + BT - 1) / BT;
+    return align_up(workspace_bytes(T, d, G, N), 256) + static_cast<size_t>(NT * TC) * BNEU * sizeof(float);
 }
 
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
-           void* workspace, cudaStream_t stream) {
+           void* workspace, cudaStream_t stream, const float* rms, float* act2) {
     CUtensorMap m_wg, m_wu, m_x, m_c;
     const cuuint64_t row_stride = static_cast<cuuint64_t>(d) * 2;
     cuuint64_t dw[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(N)};
@@ -432,6 +487,11 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
     p.units = static_cast<int64_t>(p.NT) * p.TC;
     p.status = reinterpret_cast<int*>(workspace);
     p.partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(workspace) + kWorkspaceHeader);
+    p.T = T;
+    p.rms = (rms && act2) ? rms : nullptr;
+    p.partial_act = p.rms ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(workspace) +
+                                                     align_up(workspace_bytes(T, d, G, N), 256))
+                          : nullptr;
 
     int dev = 0, sms = 0;
     DTP_CUDA_TRY(cudaGetDevice(&dev));
@@ -446,11 +506,12 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
     p.tail_items = left * p.split;
     affinity_fo_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(m_wg, m_wu, m_x, m_c, p);
     DTP_CUDA_TRY(cudaGetLastError());
-    const int64_t total = static_cast<int64_t>(G) * N;
+    const int64_t total = static_cast<int64_t>(G) * N + (p.rms ? N : 0);
     const int64_t outs_per_block = 256 / kReduceSplit;
     const int64_t want = (total + outs_per_block - 1) / outs_per_block;
     const int rblocks = static_cast<int>(want < 8 * sms ? want : 8 * sms);
-    affinity_reduce_kernel<<<rblocks, 256, 0, stream>>>(p.partial, A, G, N, p.NT, p.TC);
+    affinity_reduce_kernel<<<rblocks, 256, 0, stream>>>(p.partial, A, G, N, p.NT, p.TC, p.partial_act,
+                                                        p.rms ? act2 : nullptr);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
 }

@@ -8,15 +8,26 @@
 namespace dtp {
 namespace tc {
 size_t workspace_bytes(int64_t T, int d, int G, int N);
+size_t workspace_bytes_with_act(int64_t T, int d, int G, int N);
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
-           void* workspace, cudaStream_t stream);
+           void* workspace, cudaStream_t stream, const float* rms, float* act2);
 }  // namespace tc
 namespace f32 {
 size_t workspace_bytes(int64_t T, int d, int G, int N);
 int launch(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
-           float* A, void* workspace, cudaStream_t stream);
+           float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2);
 }  // namespace f32
+namespace sq {
+size_t down_workspace_bytes(int G, int R, int d, int N);
+int launch_down(const void* Wqkv, const void* gamma, const void* Wd, int G, int R, int d, int N, int dtype, float* bn,
+                void* workspace, cudaStream_t stream);
+size_t add_workspace_bytes(int64_t T, int G, int N);
+int launch_add(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
+               void* workspace, cudaStream_t stream);
+}  // namespace sq
 int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream);
+int launch_down_finalize(const float* act2, const float* bn, int G, int N, int64_t T_total, float* S,
+                         cudaStream_t stream);
 int launch_down_sqnorm(const void* W, int d, int N, int dtype, float* out, cudaStream_t stream);
 namespace search {
 size_t workspace_bytes(int layers, int G, int N, int D);
@@ -40,8 +51,9 @@ bool affinity_sizes_ok(int64_t T, int d, int H, int N, int dtype) {
     return true;
 }
 
-size_t affinity_ws(int64_t T, int d, int H, int N, int dtype) {
-    return dtype == DTP_BF16 ? tc::workspace_bytes(T, d, H, N) : f32::workspace_bytes(T, d, H, N);
+size_t affinity_ws(int64_t T, int d, int H, int N, int dtype, bool with_act) {
+    if (dtype != DTP_BF16) return f32::workspace_bytes(T, d, H, N);
+    return with_act ? tc::workspace_bytes_with_act(T, d, H, N) : tc::workspace_bytes(T, d, H, N);
 }
 
 bool search_sizes_ok(int layers, int H, int N, int D, int iters) {
@@ -72,25 +84,80 @@ const char* dtp_status_string(int status) {
 
 int dtp_affinity_workspace_size(int64_t T, int d, int H_kv, int N, int dtype, size_t* bytes) {
     if (!bytes || !affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
-    *bytes = affinity_ws(T, d, H_kv, N, dtype);
+    *bytes = affinity_ws(T, d, H_kv, N, dtype, true);
     return DTP_OK;
+}
+
+int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate, const void* W_up,
+                               const float* rms_next, int64_t T, int d, int H_kv, int N, int dtype, float* A,
+                               float* act2, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
+    if ((rms_next == nullptr) != (act2 == nullptr)) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;  // nothing to add; empty inputs may have null data pointers
+    if (!X || !C || !W_gate || !W_up || !A) return DTP_ERR_ARG;
+    if (!aligned16(X) || !aligned16(C) || !aligned16(W_gate) || !aligned16(W_up) || !aligned16(A))
+        return DTP_ERR_ARG;
+    const bool with_act = act2 != nullptr;
+    if (with_act && (!aligned16(act2) || !aligned16(rms_next))) return DTP_ERR_ARG;
+    const size_t need = affinity_ws(T, d, H_kv, N, dtype, with_act);
+    if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    if (dtype == DTP_BF16) return tc::launch(X, C, W_gate, W_up, T, d, H_kv, N, A, workspace, s, rms_next, act2);
+    return f32::launch(static_cast<const float*>(X), static_cast<const float*>(C), static_cast<const float*>(W_gate),
+                       static_cast<const float*>(W_up), T, d, H_kv, N, A, workspace, s, rms_next, act2);
 }
 
 int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, const void* W_up, int64_t T, int d,
                             int H_kv, int N, int dtype, float* A, void* workspace, size_t workspace_bytes,
                             void* stream) {
-    if (!affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
-    if (T == 0) return DTP_OK;  // nothing to add; empty inputs may have null data pointers
-    if (!X || !C || !W_gate || !W_up || !A) return DTP_ERR_ARG;
-    if (!aligned16(X) || !aligned16(C) || !aligned16(W_gate) || !aligned16(W_up) || !aligned16(A))
+    return dtp_affinity_accumulate_ex(X, C, W_gate, W_up, nullptr, T, d, H_kv, N, dtype, A, nullptr, workspace,
+                                      workspace_bytes, stream);
+}
+
+int dtp_affinity_add_workspace_size(int64_t T, int d, int H_kv, int N, size_t* bytes) {
+    if (!bytes || !affinity_sizes_ok(T, d, H_kv, N, DTP_BF16)) return DTP_ERR_ARG;
+    *bytes = sq::add_workspace_bytes(T, H_kv, N);
+    return DTP_OK;
+}
+
+int dtp_affinity_add_accumulate(const void* C, const void* W_gate, const void* W_up, int64_t T, int d, int H_kv,
+                                int N, float* A_add, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!affinity_sizes_ok(T, d, H_kv, N, DTP_BF16)) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;
+    if (!C || !W_gate || !W_up || !A_add || !aligned16(C) || !aligned16(W_gate) || !aligned16(W_up) ||
+        !aligned16(A_add))
         return DTP_ERR_ARG;
-    const size_t need = affinity_ws(T, d, H_kv, N, dtype);
-    if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    if (!workspace || workspace_bytes < sq::add_workspace_bytes(T, H_kv, N) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
-    if (dtype == DTP_BF16) return tc::launch(X, C, W_gate, W_up, T, d, H_kv, N, A, workspace, s);
-    return f32::launch(static_cast<const float*>(X), static_cast<const float*>(C), static_cast<const float*>(W_gate),
-                       static_cast<const float*>(W_up), T, d, H_kv, N, A, workspace, s);
+    return sq::launch_add(C, W_gate, W_up, T, d, H_kv, N, A_add, workspace, s);
+}
+
+int dtp_down_weight_workspace_size(int H_kv, int R, int d, int N, size_t* bytes) {
+    if (!bytes || H_kv < 1 || H_kv > kMaxHeads || R < 1 || d < 8 || (d % 8) || N < 1) return DTP_ERR_ARG;
+    *bytes = sq::down_workspace_bytes(H_kv, R, d, N);
+    return DTP_OK;
+}
+
+int dtp_down_weight_sqnorm(const void* Wqkv_next, const void* gamma_next, const void* W_down, int H_kv, int R, int d,
+                           int N, int dtype, float* bn, void* workspace, size_t workspace_bytes, void* stream) {
+    if (H_kv < 1 || H_kv > kMaxHeads || R < 1 || d < 8 || (d % 8) || N < 1) return DTP_ERR_ARG;
+    if (dtype != DTP_BF16) return DTP_ERR_UNSUPPORTED;
+    if (!Wqkv_next || !gamma_next || !W_down || !bn || !aligned16(Wqkv_next) || !aligned16(W_down) || !aligned16(bn))
+        return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < sq::down_workspace_bytes(H_kv, R, d, N) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    return sq::launch_down(Wqkv_next, gamma_next, W_down, H_kv, R, d, N, dtype, bn, workspace, s);
+}
+
+int dtp_down_finalize(const float* act2, const float* bn, int H_kv, int N, int64_t T_total, float* S_down,
+                      void* stream) {
+    if (!act2 || !bn || !S_down || H_kv < 1 || H_kv > kMaxHeads || N < 1 || T_total < 1) return DTP_ERR_ARG;
+    return launch_down_finalize(act2, bn, H_kv, N, T_total, S_down, static_cast<cudaStream_t>(stream));
 }
 
 int dtp_affinity_finalize(float* A, int H_kv, int N, int64_t T_total, const float* wd_sqnorm, void* stream) {

@@ -56,12 +56,21 @@ def lib():
     L.dtp_affinity_finalize.argtypes = [_vp, _i32, _i32, _i64, _vp, _vp]
     L.dtp_down_sqnorm.argtypes = [_vp, _i32, _i32, _i32, _vp, _vp]
     L.dtp_affinity_accumulate_noalloc.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp]
+    L.dtp_affinity_accumulate_ex.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _vp,
+                                             _sz, _vp]
+    L.dtp_affinity_add_workspace_size.argtypes = [_i64, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_affinity_add_accumulate.argtypes = [_vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
+    L.dtp_down_weight_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_down_weight_sqnorm.argtypes = [_vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
+    L.dtp_down_finalize.argtypes = [_vp, _vp, _i32, _i32, _i64, _vp, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_search_layout_batched.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                             _vp]
-    for fn in ("dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
+    for fn in ("dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
+               "dtp_down_weight_workspace_size", "dtp_down_weight_sqnorm", "dtp_down_finalize",
+               "dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
                "dtp_affinity_finalize",
                "dtp_down_sqnorm", "dtp_workspace_status", "dtp_search_workspace_size", "dtp_search_layout",
                "dtp_search_layout_batched"):
@@ -136,6 +145,82 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
                                        _ptr(workspace), workspace.numel(), _stream(stream))
     _check("dtp_affinity_accumulate", st)
     return A
+
+
+def affinity_accumulate_down(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
+                             rms_next: torch.Tensor, A: torch.Tensor | None = None, act2: torch.Tensor | None = None,
+                             workspace: torch.Tensor | None = None, stream=None):
+    """The affinity pass plus the down-edge activation term (Sec. 3).
+
+    A[h,k] += sum_t Delta^2 as in affinity_accumulate, and act2[k] += sum_t
+    (silu(g_k) u_k)^2 / rms_next[t]^2 with rms_next [T] fp32 the rms of the
+    residual entering the next layer's pre-norm.  Returns (A, act2).
+    """
+    T, d = X.shape
+    H = C.shape[0]
+    N = W_gate.shape[0]
+    code = _dtype_code(X)
+    if A is None:
+        A = torch.zeros((H, N), dtype=torch.float32, device=X.device)
+    if act2 is None:
+        act2 = torch.zeros(N, dtype=torch.float32, device=X.device)
+    if rms_next.shape != (T,) or rms_next.dtype != torch.float32:
+        raise ValueError("rms_next must be fp32 [T]")
+    if workspace is None:
+        workspace = affinity_workspace(T, d, H, N, code, X.device)
+    st = lib().dtp_affinity_accumulate_ex(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), _ptr(rms_next), T, d, H, N,
+                                          code, _ptr(A), _ptr(act2), _ptr(workspace), workspace.numel(),
+                                          _stream(stream))
+    _check("dtp_affinity_accumulate_ex", st)
+    return A, act2
+
+
+def affinity_add_accumulate(C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
+                            A_add: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                            stream=None) -> torch.Tensor:
+    """ADD score before the mean (Sec. 3): A_add[h,k] += sum_t (p_h.w^g_k)^2 + (p_h.w^u_k)^2; bf16 inputs."""
+    H, T, d = C.shape
+    N = W_gate.shape[0]
+    if A_add is None:
+        A_add = torch.zeros((H, N), dtype=torch.float32, device=C.device)
+    if workspace is None:
+        n = _sz(0)
+        _check("dtp_affinity_add_workspace_size", lib().dtp_affinity_add_workspace_size(T, d, H, N, ctypes.byref(n)))
+        workspace = torch.empty(n.value, dtype=torch.uint8, device=C.device)
+    st = lib().dtp_affinity_add_accumulate(_ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, _ptr(A_add),
+                                           _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_affinity_add_accumulate", st)
+    return A_add
+
+
+def down_weight_sqnorm(Wqkv_next: torch.Tensor, gamma_next: torch.Tensor, W_down: torch.Tensor,
+                       workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """||b_gk||^2 = ||W^qkv_g (gamma' . w^d_k)||^2 (Sec. 3, down edge) -> fp32 [H_kv, N].
+
+    Wqkv_next [H_kv, R, d]: the next layer's q/k/v rows of each KV group;
+    gamma_next [d]: its pre-norm gain; W_down [d, N].  All bf16.
+    """
+    H, R, d = Wqkv_next.shape
+    N = W_down.shape[1]
+    bn = torch.empty((H, N), dtype=torch.float32, device=W_down.device)
+    if workspace is None:
+        n = _sz(0)
+        _check("dtp_down_weight_workspace_size", lib().dtp_down_weight_workspace_size(H, R, d, N, ctypes.byref(n)))
+        workspace = torch.empty(n.value, dtype=torch.uint8, device=W_down.device)
+    st = lib().dtp_down_weight_sqnorm(_ptr(Wqkv_next), _ptr(gamma_next), _ptr(W_down), H, R, d, N,
+                                      _dtype_code(W_down), _ptr(bn), _ptr(workspace), workspace.numel(),
+                                      _stream(stream))
+    _check("dtp_down_weight_sqnorm", st)
+    return bn
+
+
+def down_finalize(act2: torch.Tensor, bn: torch.Tensor, T_total: int, stream=None) -> torch.Tensor:
+    """S_down[g,k] = act2[k] / T_total * bn[g,k] (Sec. 3), stored [H_kv, N]."""
+    H, N = bn.shape
+    S = torch.empty((H, N), dtype=torch.float32, device=bn.device)
+    _check("dtp_down_finalize", lib().dtp_down_finalize(_ptr(act2), _ptr(bn), H, N, int(T_total), _ptr(S),
+                                                        _stream(stream)))
+    return S
 
 
 def affinity_accumulate_noalloc(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,

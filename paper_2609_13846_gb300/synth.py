@@ -132,3 +132,23 @@ def make_affinity_matrix(G: int, N: int, seed: int, *, kind: str = "lognormal", 
     if kind == "zeros":
         return torch.zeros((G, N), device=device, dtype=torch.float32)
     raise ValueError(kind)
+
+
+def make_down_inputs(d: int, G: int, R: int, N: int, T: int, seed: int, *, dtype: str = "bf16", device="cpu"):
+    """Seeded stand-ins for the next layer's side of the down edge (Sec. 3).
+
+    Wqkv [G, R, d]: the next layer's q/k/v rows of each KV group, N(0, 0.02^2);
+    gamma [d]: its pre-norm gain, 1 + N(0, 0.1^2); W_down [d, N]: this layer's
+    down projection, N(0, 0.02^2); rms [T] fp32: the rms of the residual entering
+    the next pre-norm, uniform in [0.5, 1.5].  Draw order as listed.
+    """
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed))
+    out = dict(Wqkv=_randn(gen, (G, R, d), device) * 0.02,
+               gamma=1.0 + 0.1 * _randn(gen, (d,), device),
+               W_down=_randn(gen, (d, N), device) * 0.02)
+    rms = 0.5 + torch.rand((T,), generator=gen, device=device, dtype=torch.float32)
+    if dtype == "bf16":
+        out = {k: v.to(torch.bfloat16) for k, v in out.items()}
+    out["rms"] = rms
+    return out

@@ -202,3 +202,24 @@ def test_synthetic_recipe_shapes_and_scales():
     ratio = torch.linalg.vector_norm(C.reshape(4, -1), dim=1) / torch.linalg.vector_norm(X)
     assert torch.all(ratio >= 0.1 - 1e-5) and torch.all(ratio <= 1.0 + 1e-5)
     assert abs(float(L["W_gate"].std()) - 0.02) < 2e-3
+
+
+def test_add_score_is_the_removed_pre_activation_change():
+    """ADD (Sec. 3): removing head h's piece changes neuron k's gate and up pre-activations by
+    exactly p_h . w (they are linear); the score is the summed square of both changes."""
+    X, C, Wg, Wu = _tiny(seed=14)
+    A = oracle.affinity_add(C, Wg, Wu)
+    for h in range(C.shape[0]):
+        dg = X @ Wg.T - (X - C[h]) @ Wg.T
+        du = X @ Wu.T - (X - C[h]) @ Wu.T
+        np.testing.assert_allclose(A[h], (dg ** 2 + du ** 2).sum(0), rtol=1e-10)
+
+
+def test_add_score_ignores_the_operating_point_and_fo_does_not():
+    """ADD does not depend on X; FO does (Sec. 3: ADD ignores the operating point of the nonlinearity)."""
+    X, C, Wg, Wu = _tiny(seed=15)
+    A1 = oracle.affinity_add(C, Wg, Wu)
+    assert np.array_equal(A1, oracle.affinity_add(C, Wg, Wu))
+    F1 = oracle.affinity_fo(X, C, Wg, Wu)
+    F2 = oracle.affinity_fo(2.0 * X, C, Wg, Wu)
+    assert np.max(np.abs(F1 - F2)) > 1e-3 * np.max(F1)
