@@ -259,6 +259,39 @@ int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D
                               double* score, int32_t* iters_done, void* workspace,
                               size_t workspace_bytes, void* stream);
 
+/*
+ * The whole-model objective of Sec. 3 (Eq. objective, both sums) and its
+ * optimiser over `layers` layers:
+ *   J(h, nu) = sum_i sum over (g,k) with h_i(g) == nu_i(k) of S_up_i[g,k] / sum S_up_i
+ *            + sum_{i<layers-1} sum over (g,k) with nu_i(k) == h_{i+1}(g) of
+ *                                               S_down_i[g,k] / sum S_down_i
+ * J lies in [0, 2*layers - 1]; a uniform random balanced layout scores
+ * (2*layers - 1)/D in expectation.
+ *   - Exact arithmetic: each matrix is mapped to n = floor(q 2^39 / sum q),
+ *     q = floor(S 2^(24-e)), max(S) < 2^e; J_q = sum of co-located n.
+ *   - Start: contiguous heads in every layer.  One iteration: every layer's
+ *     neuron step given all head partitions (gain M_kl of Sec. 3 with the up
+ *     term from h_i and the down term from h_{i+1}), then every layer's head
+ *     step given all neuron assignments (up term over nu_i, down term over
+ *     nu_{i-1}).  Each step maximises J exactly given the other block.
+ *   - Ties: lexicographically smallest nu_i and h_i, as in dtp_search_layout.
+ *   - Stop after `iters` iterations or the first without a strict increase.
+ *
+ *   S_up       [layers, H_kv, N] fp32, device, finite and >= 0
+ *   S_down     [layers-1, H_kv, N] fp32 (S_down[i][g,k]: group g of layer i+1
+ *              on neuron k of layer i; dtp_down_finalize's layout), or NULL
+ *              when layers == 1
+ *   head_part  [layers, H_kv] int32 out; neuron_dev [layers, N] int32 out
+ *   J_q        int64 out, J in units of 2^-39; J double out; iters_done int32 out
+ * Same size rules as dtp_search_layout; workspace from
+ * dtp_search_chain_workspace_size.  Asynchronous; invalid entries or loop
+ * limits are reported through the workspace status word.
+ */
+int dtp_search_chain_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes);
+int dtp_search_chain(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D,
+                     int iters, int32_t* head_part, int32_t* neuron_dev, int64_t* J_q, double* J,
+                     int32_t* iters_done, void* workspace, size_t workspace_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -34,6 +34,9 @@ size_t workspace_bytes(int layers, int G, int N, int D);
 int64_t partition_count(int G, int D);
 int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* head, int32_t* nu, int64_t* score_q,
            double* score, int32_t* iters_done, void* workspace, cudaStream_t stream);
+size_t chain_workspace_bytes(int Lyr, int G, int N, int D);
+int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters, int32_t* head,
+                 int32_t* nu, int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream);
 }  // namespace search
 }  // namespace dtp
 
@@ -195,6 +198,25 @@ int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D
     if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
     return search::launch(A, layers, H_kv, N, D, iters, head_part, neuron_dev, score_q, score, iters_done, workspace,
                           static_cast<cudaStream_t>(stream));
+}
+
+int dtp_search_chain_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes) {
+    if (!bytes || !search_sizes_ok(layers, H_kv, N, D, 1)) return DTP_ERR_ARG;
+    *bytes = search::chain_workspace_bytes(layers, H_kv, N, D);
+    return DTP_OK;
+}
+
+int dtp_search_chain(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D, int iters,
+                     int32_t* head_part, int32_t* neuron_dev, int64_t* J_q, double* J, int32_t* iters_done,
+                     void* workspace, size_t workspace_bytes, void* stream) {
+    if (!search_sizes_ok(layers, H_kv, N, D, iters)) return DTP_ERR_ARG;
+    if (!S_up || (layers > 1 && !S_down) || !head_part || !neuron_dev || !J_q || !J || !iters_done)
+        return DTP_ERR_ARG;
+    if (!aligned16(S_up) || (S_down && !aligned16(S_down))) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < search::chain_workspace_bytes(layers, H_kv, N, D) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
+    return search::launch_chain(S_up, S_down, layers, H_kv, N, D, iters, head_part, neuron_dev, J_q, J, iters_done,
+                                workspace, static_cast<cudaStream_t>(stream));
 }
 
 int dtp_search_layout(const float* A, int H_kv, int N, int D, int iters, int32_t* head_part, int32_t* neuron_dev,

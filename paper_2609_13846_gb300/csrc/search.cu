@@ -60,6 +60,7 @@ struct Shared {
     long long sel_rank;
     int64_t total, J, Jprev;
     int h[GMAX];
+    int hn[GMAX];                  // next layer's head partition (whole-model search)
     int status;
     int flag;
     int kstar;
@@ -70,8 +71,8 @@ struct Shared {
 
 __device__ __forceinline__ size_t align_up_dev(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// floor(a * 2^(40-e)) for a finite a >= 0, by shifting the fp32 significand.
-__device__ __forceinline__ int64_t quantize(float a, int e) {
+// floor(a * 2^(bits-e)) for a finite a >= 0, by shifting the fp32 significand.
+__device__ __forceinline__ int64_t quantize_bits(float a, int e, int bits) {
     const uint32_t b = __float_as_uint(a);
     const uint32_t ex = (b >> 23) & 0xFFu;
     uint64_t m = b & 0x7FFFFFu;
@@ -82,11 +83,13 @@ __device__ __forceinline__ int64_t quantize(float a, int e) {
         m |= 0x800000u;
         E = static_cast<int>(ex) - 150;
     }
-    const int s = E + kFixedBits - e;
+    const int s = E + bits - e;
     if (s >= 0) return static_cast<int64_t>(m << s);
     if (s <= -40) return 0;
     return static_cast<int64_t>(m >> (-s));
 }
+
+__device__ __forceinline__ int64_t quantize(float a, int e) { return quantize_bits(a, e, kFixedBits); }
 
 __device__ __forceinline__ uint64_t pack_gain(int64_t v, int k) {
     return (static_cast<uint64_t>(v + kValBias) << kIdxBits) |
@@ -492,8 +495,9 @@ __device__ __forceinline__ void better(int64_t& s, int& i, int64_t s2, int i2) {
     if (s2 > s || (s2 == s && i2 < i)) s = s2, i = i2;
 }
 
+// Head-step column sums of one layer: B[g,l] = sum over neurons k on device l of q[g,k].
 template <int DT>
-__device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
+__device__ void head_sums(const Layer& L, Shared& sh) {
     const int G = L.G, D = L.D;
     if (threadIdx.x < GMAX * DMAX) sh.B[threadIdx.x] = 0;
     __syncthreads();
@@ -523,7 +527,15 @@ __device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
         }
     }
     __syncthreads();
-    // score every labelled partition; each thread a contiguous range in lexicographic order
+}
+
+// The best labelled balanced partition for the column sums in sh.B: every
+// partition scored by a slice of the block, each thread a contiguous range in
+// lexicographic order; result (lexicographically smallest among ties) in
+// sh.h, its score in sh.J.
+__device__ void choose_partition(const Layer& L, Shared& sh, uint32_t n_parts) {
+    const int G = L.G, D = L.D;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t lo = static_cast<uint32_t>((static_cast<uint64_t>(n_parts) * threadIdx.x) / kThreads);
     const uint32_t hi = static_cast<uint32_t>((static_cast<uint64_t>(n_parts) * (threadIdx.x + 1)) / kThreads);
     int64_t best = kNegInf;
@@ -561,6 +573,12 @@ __device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
         }
     }
     __syncthreads();
+}
+
+template <int DT>
+__device__ void head_step(const Layer& L, Shared& sh, uint32_t n_parts) {
+    head_sums<DT>(L, sh);
+    choose_partition(L, sh, n_parts);
 }
 
 // ------------------------------------------------------------------ kernel --
@@ -657,6 +675,211 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     }
 }
 
+// ------------------------------------------------------- whole-model search --
+//
+// Eq. objective with both sums: J = sum_i up_i + sum_{i<L-1} down_i, each matrix
+// in its exact unit-mass form n = floor(floor(S 2^(24-e)) 2^39 / total).  One
+// iteration = every layer's neuron step given all head partitions (gain from
+// h_i for the up edge and h_{i+1} for the down edge), then every layer's head
+// step given all neuron assignments (column sums over nu_i for the up edge and
+// nu_{i-1} for the down edge), then the score.  Each step maximises J exactly
+// given the other block, so layers run in parallel, one block each.  A device
+// flag stops later iterations after the first one without a strict increase,
+// so the host never waits.
+
+constexpr int kNormBits = 39;
+constexpr int kNormPreBits = 24;
+
+struct ChainState {
+    int done;
+    int iters;
+    int64_t prev;
+};
+
+__global__ void chain_init_kernel(ChainState* st, int64_t* J_q, double* J, int32_t* iters_done) {
+    st->done = 0;
+    st->iters = 0;
+    st->prev = -1;
+    *J_q = 0;
+    *J = 0.0;
+    *iters_done = 0;
+}
+
+// One block per matrix: m < L is the up edge of layer m, m >= L the down edge of layer m - L.
+__global__ void __launch_bounds__(kThreads, 1)
+chain_normalize_kernel(const float* __restrict__ S_up, const float* __restrict__ S_down, int L, int G, int N, int D,
+                       int64_t* __restrict__ nbuf, int32_t* __restrict__ head, ChainState* st, int* ws_status) {
+    __shared__ Shared sh;
+    const int m = blockIdx.x;
+    const int64_t GN = static_cast<int64_t>(G) * N;
+    const float* src = m < L ? S_up + m * GN : S_down + (m - L) * GN;
+    int64_t* dst = nbuf + m * GN;
+    if (m < L && threadIdx.x < G) head[m * G + threadIdx.x] = (threadIdx.x * D) / G;
+    uint32_t amax_bits = 0;
+    int bad = 0;
+    for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
+        const float a = src[i];
+        if (!(a >= 0.0f) || isinf(a)) bad = 1;
+        else amax_bits = max(amax_bits, __float_as_uint(a));
+    }
+    bad = __syncthreads_or(bad);
+    const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
+    if (bad) {
+        if (threadIdx.x == 0) {
+            atomicMin(ws_status, static_cast<int>(DTP_ERR_ARG));
+            st->done = 1;
+        }
+        return;
+    }
+    const float amax = __uint_as_float(static_cast<uint32_t>(amax_all));
+    int e = 0;
+    if (amax > 0.0f) frexpf(amax, &e);
+    int64_t part = 0;
+    for (int64_t i = threadIdx.x; i < GN; i += kThreads) part += quantize_bits(src[i], e, kNormPreBits);
+    const uint64_t total = static_cast<uint64_t>(block_sum_i64(part, sh));
+    for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
+        const uint64_t q = static_cast<uint64_t>(quantize_bits(src[i], e, kNormPreBits));
+        dst[i] = total ? static_cast<int64_t>((q << kNormBits) / total) : 0;
+    }
+}
+
+// M[k,l] = up mass of k from heads of layer i on l + down mass of k into heads of layer i+1 on l.
+template <int DT>
+__device__ void build_gain_chain(const Layer& L, Shared& sh, const int64_t* __restrict__ nU,
+                                 const int64_t* __restrict__ nD) {
+    for (int k = threadIdx.x; k < L.N; k += kThreads) {
+        int64_t m[DT];
+#pragma unroll
+        for (int l = 0; l < DT; ++l) m[l] = 0;
+        for (int g = 0; g < L.G; ++g) {
+            const int64_t u = nU[static_cast<int64_t>(g) * L.N + k];
+            const int64_t dn = nD ? nD[static_cast<int64_t>(g) * L.N + k] : 0;
+            const int hg = sh.h[g], hn = nD ? sh.hn[g] : -1;
+#pragma unroll
+            for (int l = 0; l < DT; ++l) m[l] += (l == hg ? u : 0) + (l == hn ? dn : 0);
+        }
+#pragma unroll
+        for (int l = 0; l < DT; ++l) L.M[static_cast<int64_t>(k) * DT + l] = m[l];
+    }
+    __syncthreads();
+}
+
+// B[g,l] = up mass of g on device l under nu_i + down mass into g from neurons of layer i-1 on l.
+template <int DT>
+__device__ void head_sums_chain(const Layer& L, Shared& sh, const int64_t* __restrict__ nU,
+                                const int32_t* __restrict__ nu_i, const int64_t* __restrict__ nD,
+                                const int32_t* __restrict__ nu_prev) {
+    const int G = L.G;
+    if (threadIdx.x < GMAX * DMAX) sh.B[threadIdx.x] = 0;
+    __syncthreads();
+    const int warps_per_head = kWarps / G;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = warp / warps_per_head;
+    if (g < G) {
+        const int tph = warps_per_head * 32;
+        const int sub = (warp % warps_per_head) * 32 + lane;
+        int64_t acc[DT];
+#pragma unroll
+        for (int l = 0; l < DT; ++l) acc[l] = 0;
+        for (int k = sub; k < L.N; k += tph) {
+            const int64_t u = nU[static_cast<int64_t>(g) * L.N + k];
+            const int lu = nu_i[k];
+            const int64_t dn = nD ? nD[static_cast<int64_t>(g) * L.N + k] : 0;
+            const int ld = nD ? nu_prev[k] : -1;
+#pragma unroll
+            for (int l = 0; l < DT; ++l) acc[l] += (l == lu ? u : 0) + (l == ld ? dn : 0);
+        }
+#pragma unroll
+        for (int l = 0; l < DT; ++l) {
+            const int64_t v = warp_sum_i64(acc[l]);
+            if (lane == 0 && v)
+                atomicAdd(reinterpret_cast<unsigned long long*>(&sh.B[g * DT + l]), static_cast<unsigned long long>(v));
+        }
+    }
+    __syncthreads();
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads, 1)
+chain_neuron_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, const int32_t* __restrict__ head,
+                    int32_t* __restrict__ nu_out, int64_t* __restrict__ prices, ChainState* st, int* ws_status,
+                    uint8_t* __restrict__ gbuf, size_t per_layer, int use_smem) {
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ Shared sh;
+    if (*reinterpret_cast<volatile int*>(&st->done)) return;
+    const int i = blockIdx.x;
+    const int64_t GN = static_cast<int64_t>(G) * N;
+    uint8_t* buf = use_smem ? dsm : gbuf + static_cast<size_t>(i) * per_layer;
+    Layer L;
+    L.A = nullptr;
+    L.G = G;
+    L.N = N;
+    L.D = DT;
+    L.cap = N / DT;
+    L.e = 0;
+    L.M = reinterpret_cast<int64_t*>(buf);
+    L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * DT * sizeof(int64_t));
+    const bool has_down = i + 1 < Lyr;
+    if (threadIdx.x < G) {
+        sh.h[threadIdx.x] = head[i * G + threadIdx.x];
+        sh.hn[threadIdx.x] = has_down ? head[(i + 1) * G + threadIdx.x] : -1;
+    }
+    if (threadIdx.x < DMAX) sh.pi[threadIdx.x] = prices[i * DMAX + threadIdx.x];
+    if (threadIdx.x == 0) sh.status = DTP_OK;
+    __syncthreads();
+    build_gain_chain<DT>(L, sh, nbuf + i * GN, has_down ? nbuf + (Lyr + i) * GN : nullptr);
+    if constexpr (DT == 2) neuron_step_d2(L, sh);
+    else neuron_step_general<DT>(L, sh);
+    __syncthreads();
+    if (sh.status != DTP_OK) {
+        if (threadIdx.x == 0) {
+            atomicMin(ws_status, sh.status);
+            st->done = 1;
+        }
+        return;
+    }
+    for (int k = threadIdx.x; k < N; k += kThreads) nu_out[static_cast<int64_t>(i) * N + k] = L.nu[k];
+    if (threadIdx.x < DMAX) prices[i * DMAX + threadIdx.x] = sh.pi[threadIdx.x];
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads, 1)
+chain_head_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, const int32_t* __restrict__ nu_all,
+                  int32_t* __restrict__ head, int64_t* __restrict__ layer_score, ChainState* st, uint32_t n_parts) {
+    __shared__ Shared sh;
+    if (*reinterpret_cast<volatile int*>(&st->done)) return;
+    const int i = blockIdx.x;
+    const int64_t GN = static_cast<int64_t>(G) * N;
+    Layer L;
+    L.A = nullptr;
+    L.G = G;
+    L.N = N;
+    L.D = DT;
+    L.cap = N / DT;
+    L.e = 0;
+    L.M = nullptr;
+    L.nu = nullptr;
+    head_sums_chain<DT>(L, sh, nbuf + i * GN, nu_all + static_cast<int64_t>(i) * N,
+                        i > 0 ? nbuf + (Lyr + i - 1) * GN : nullptr,
+                        i > 0 ? nu_all + static_cast<int64_t>(i - 1) * N : nullptr);
+    choose_partition(L, sh, n_parts);
+    if (threadIdx.x < G) head[i * G + threadIdx.x] = sh.h[threadIdx.x];
+    if (threadIdx.x == 0) layer_score[i] = sh.J;
+}
+
+__global__ void chain_score_kernel(int Lyr, const int64_t* __restrict__ layer_score, ChainState* st, int64_t* J_q,
+                                   double* J, int32_t* iters_done) {
+    if (threadIdx.x != 0 || st->done) return;
+    int64_t total = 0;
+    for (int i = 0; i < Lyr; ++i) total += layer_score[i];
+    st->iters += 1;
+    *iters_done = st->iters;
+    *J_q = total;
+    *J = ldexp(static_cast<double>(total), -kNormBits);
+    if (total <= st->prev) st->done = 1;
+    else st->prev = total;
+}
+
 // --------------------------------------------------------------------- host --
 
 int64_t partition_count(int G, int D) {
@@ -711,6 +934,81 @@ int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* 
                                                       per_layer_bytes(N, D), mode);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
+}
+
+}  // namespace search
+}  // namespace dtp
+
+namespace dtp {
+namespace search {
+
+static size_t chain_layout(int Lyr, int G, int N, int D, size_t* off_state, size_t* off_score, size_t* off_prices,
+                           size_t* off_nbuf, size_t* off_gbuf) {
+    const size_t GN = static_cast<size_t>(G) * N;
+    size_t o = kWorkspaceHeader;
+    *off_state = o;
+    o += 256;
+    *off_score = o;
+    o += align_up(static_cast<size_t>(Lyr) * sizeof(int64_t), 256);
+    *off_prices = o;
+    o += align_up(static_cast<size_t>(Lyr) * DMAX * sizeof(int64_t), 256);
+    *off_nbuf = o;
+    o += align_up(static_cast<size_t>(2 * Lyr - 1) * GN * sizeof(int64_t), 256);
+    *off_gbuf = o;
+    if (!fits_smem(N, D)) o += static_cast<size_t>(Lyr) * per_layer_bytes(N, D);
+    return o;
+}
+
+size_t chain_workspace_bytes(int Lyr, int G, int N, int D) {
+    size_t a, b, c, d, e;
+    return chain_layout(Lyr, G, N, D, &a, &b, &c, &d, &e);
+}
+
+template <int DT>
+static int launch_chain_t(const float* S_up, const float* S_down, int Lyr, int G, int N, int iters, int32_t* head,
+                          int32_t* nu, int64_t* J_q, double* J, int32_t* iters_done, uint8_t* ws,
+                          cudaStream_t stream) {
+    size_t o_state, o_score, o_prices, o_nbuf, o_gbuf;
+    chain_layout(Lyr, G, N, DT, &o_state, &o_score, &o_prices, &o_nbuf, &o_gbuf);
+    int* ws_status = reinterpret_cast<int*>(ws);
+    ChainState* st = reinterpret_cast<ChainState*>(ws + o_state);
+    int64_t* layer_score = reinterpret_cast<int64_t*>(ws + o_score);
+    int64_t* prices = reinterpret_cast<int64_t*>(ws + o_prices);
+    int64_t* nbuf = reinterpret_cast<int64_t*>(ws + o_nbuf);
+    uint8_t* gbuf = ws + o_gbuf;
+    const bool smem = fits_smem(N, DT);
+    const size_t dyn = smem ? per_layer_bytes(N, DT) : 0;
+    DTP_CUDA_TRY(cudaFuncSetAttribute(chain_neuron_kernel<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kSmemBudget)));
+    DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
+    DTP_CUDA_TRY(cudaMemsetAsync(prices, 0, static_cast<size_t>(Lyr) * DMAX * sizeof(int64_t), stream));
+    chain_init_kernel<<<1, 1, 0, stream>>>(st, J_q, J, iters_done);
+    chain_normalize_kernel<<<2 * Lyr - 1, kThreads, 0, stream>>>(S_up, S_down, Lyr, G, N, DT, nbuf, head, st,
+                                                                 ws_status);
+    const uint32_t n_parts = static_cast<uint32_t>(partition_count(G, DT));
+    for (int it = 0; it < iters; ++it) {
+        chain_neuron_kernel<DT><<<Lyr, kThreads, dyn, stream>>>(Lyr, G, N, nbuf, head, nu, prices, st, ws_status, gbuf,
+                                                                 per_layer_bytes(N, DT), smem ? 1 : 0);
+        chain_head_kernel<DT><<<Lyr, kThreads, 0, stream>>>(Lyr, G, N, nbuf, nu, head, layer_score, st, n_parts);
+        chain_score_kernel<<<1, 32, 0, stream>>>(Lyr, layer_score, st, J_q, J, iters_done);
+    }
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
+}
+
+int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters, int32_t* head,
+                 int32_t* nu, int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream) {
+    uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+    switch (D) {
+        case 2: return launch_chain_t<2>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        case 3: return launch_chain_t<3>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        case 4: return launch_chain_t<4>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        case 5: return launch_chain_t<5>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        case 6: return launch_chain_t<6>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        case 7: return launch_chain_t<7>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        case 8: return launch_chain_t<8>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        default: return DTP_ERR_ARG;
+    }
 }
 
 }  // namespace search

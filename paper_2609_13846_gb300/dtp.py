@@ -63,12 +63,14 @@ def lib():
     L.dtp_down_weight_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_down_weight_sqnorm.argtypes = [_vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
     L.dtp_down_finalize.argtypes = [_vp, _vp, _i32, _i32, _i64, _vp, _vp]
+    L.dtp_search_chain_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_search_chain.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_search_layout_batched.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                             _vp]
-    for fn in ("dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
+    for fn in ("dtp_search_chain_workspace_size", "dtp_search_chain", "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
                "dtp_down_weight_workspace_size", "dtp_down_weight_sqnorm", "dtp_down_finalize",
                "dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
                "dtp_affinity_finalize",
@@ -306,3 +308,35 @@ def search_layout(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor |
     """Coordinate ascent on one layer's A [H_kv, N]; tensors as in search_layout_batched, unbatched."""
     r = search_layout_batched(A.unsqueeze(0) if A.dim() == 2 else A, D, iters, workspace, stream, check)
     return {k: v[0] for k, v in r.items()}
+
+
+def search_chain(S_up: torch.Tensor, S_down: torch.Tensor | None, D: int, iters: int,
+                 workspace: torch.Tensor | None = None, stream=None, check: bool = True) -> dict:
+    """Coordinate ascent on the whole-model objective (Sec. 3, Eq. objective, up and down edges).
+
+    S_up [L, H_kv, N], S_down [L-1, H_kv, N] (None when L == 1), fp32 CUDA.
+    Returns device tensors: h [L,H_kv] int32, nu [L,N] int32, J_q int64 (units
+    of 2^-39), J float64, iters_done int32.  Asynchronous unless ``check``.
+    """
+    if S_up.dtype != torch.float32 or not S_up.is_cuda or not S_up.is_contiguous():
+        raise ValueError("S_up must be a contiguous fp32 CUDA tensor [L, H_kv, N]")
+    Lyr, H, N = S_up.shape
+    if Lyr > 1 and (S_down is None or S_down.shape != (Lyr - 1, H, N) or not S_down.is_contiguous()):
+        raise ValueError("S_down must be a contiguous fp32 tensor [L-1, H_kv, N]")
+    dev = S_up.device
+    out = dict(h=torch.empty((Lyr, H), dtype=torch.int32, device=dev),
+               nu=torch.empty((Lyr, N), dtype=torch.int32, device=dev),
+               J_q=torch.empty((), dtype=torch.int64, device=dev),
+               J=torch.empty((), dtype=torch.float64, device=dev),
+               iters_done=torch.empty((), dtype=torch.int32, device=dev))
+    if workspace is None:
+        n = _sz(0)
+        _check("dtp_search_chain_workspace_size", lib().dtp_search_chain_workspace_size(Lyr, H, N, D, ctypes.byref(n)))
+        workspace = torch.empty(n.value, dtype=torch.uint8, device=dev)
+    st = lib().dtp_search_chain(_ptr(S_up), _ptr(S_down) if Lyr > 1 else None, Lyr, H, N, D, iters, _ptr(out["h"]),
+                                _ptr(out["nu"]), _ptr(out["J_q"]), _ptr(out["J"]), _ptr(out["iters_done"]),
+                                _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_search_chain", st)
+    if check:
+        _check("dtp_search_chain (device status)", workspace_status(workspace, stream))
+    return out
