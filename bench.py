@@ -188,6 +188,66 @@ def cpu_baseline(w, A_gpu, budget_s: float):
             "search_ms": 1e3 * t_search}
 
 
+def run_model(args):
+    """Whole-model pipeline timing: every layer's affinity pass with the down-edge term on all
+    its tokens, the ||w^d||^2 finalize, ||b_gk||^2 and S_down, then the whole-model search per D.
+    Inputs are drawn per layer on the device outside the timed intervals."""
+    from paper_2609_13846_gb300 import dtp
+    w = synth.WORKLOADS[args.model]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    Lyr, G, N, T, d = w.layers, w.G, w.N, w.T, w.d
+    S_up = torch.empty((Lyr, G, N), dtype=torch.float32, device=dev)
+    S_down = torch.empty((max(Lyr - 1, 1), G, N), dtype=torch.float32, device=dev)
+    ws = dtp.affinity_workspace(T, d, G, N, dtp.DTP_BF16, dev)
+    t_aff = t_down = 0.0
+    for i in range(Lyr):
+        L = synth.make_workload_layer(w, i, device=dev)
+        Dn = synth.make_down_inputs(d, G, w.qkv_rows, N, T, seed=w.seed + 1000 + i, device=dev)
+        act2 = torch.zeros(N, dtype=torch.float32, device=dev)
+        A = S_up[i]
+        A.zero_()
+        torch.cuda.synchronize()
+        e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        e0.record(stream)
+        dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"], A=A, act2=act2, workspace=ws)
+        dtp.affinity_finalize(A, T, dtp.down_sqnorm(Dn["W_down"]))
+        e1.record(stream)
+        if i + 1 < Lyr:
+            bn = dtp.down_weight_sqnorm(Dn["Wqkv"], Dn["gamma"], Dn["W_down"])
+            S_down[i].copy_(dtp.down_finalize(act2, bn, T))
+        e2.record(stream)
+        torch.cuda.synchronize()
+        t_aff += e0.elapsed_time(e1)
+        t_down += e1.elapsed_time(e2)
+        del L, Dn
+    if dtp.workspace_status(ws) != dtp.DTP_OK:
+        raise RuntimeError("affinity kernel reported a device-side error")
+    searches = {}
+    for D in w.D:
+        r = dtp.search_chain(S_up, S_down if Lyr > 1 else None, D, w.iters)
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(3):
+            r = dtp.search_chain(S_up, S_down if Lyr > 1 else None, D, w.iters, check=False)
+        s1.record(stream)
+        torch.cuda.synchronize()
+        searches[f"D{D}"] = {"ms": s0.elapsed_time(s1) / 3, "J": float(r["J"]), "J_random": (2 * Lyr - 1) / D,
+                             "iters_done": int(r["iters_done"])}
+    total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values())
+    fl = 2.0 * d * 2 * N * (G + 1) * T * Lyr
+    line = {"metric": f"whole-model affinity + layout time ({args.model})", "value": total_ms / 1e3, "unit": "s",
+            "higher_is_better": False, "n_gpus": 1, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.model, "layers": Lyr, "d": d, "G": G, "N": N, "T_per_layer": T,
+                       "D": list(w.D), "iters": w.iters, "qkv_rows": w.qkv_rows},
+            "affinity_ms": t_aff, "affinity_tflops": fl / (t_aff / 1e3) / 1e12,
+            "layer_tokens_per_s": Lyr * T / (t_aff / 1e3), "down_edge_ms": t_down, "search": searches,
+            "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -197,8 +257,12 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--cpu-tokens", type=int, default=64, help="token slice per step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--model", default=None, help="time a whole-model pipeline instead, e.g. qwen3_0.6b_model")
     args = ap.parse_args()
     w = synth.WORKLOADS[WORKLOAD]
+    if args.model:
+        run_model(args)
+        return
 
     if args.impl == "reference":
         run_reference(args, w)

@@ -267,8 +267,9 @@ int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D
  *                                               S_down_i[g,k] / sum S_down_i
  * J lies in [0, 2*layers - 1]; a uniform random balanced layout scores
  * (2*layers - 1)/D in expectation.
- *   - Exact arithmetic: each matrix is mapped to n = floor(q 2^39 / sum q),
- *     q = floor(S 2^(24-e)), max(S) < 2^e; J_q = sum of co-located n.
+ *   - Exact arithmetic: each matrix is mapped to n = floor(q 2^43 / sum q),
+ *     q = floor(S 2^(40-e)), max(S) < 2^e (the product in 128 bits); J_q =
+ *     sum of co-located n.
  *   - Start: contiguous heads in every layer.  One iteration: every layer's
  *     neuron step given all head partitions (gain M_kl of Sec. 3 with the up
  *     term from h_i and the down term from h_{i+1}), then every layer's head
@@ -282,7 +283,7 @@ int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D
  *              on neuron k of layer i; dtp_down_finalize's layout), or NULL
  *              when layers == 1
  *   head_part  [layers, H_kv] int32 out; neuron_dev [layers, N] int32 out
- *   J_q        int64 out, J in units of 2^-39; J double out; iters_done int32 out
+ *   J_q        int64 out, J in units of 2^-43; J double out; iters_done int32 out
  * Same size rules as dtp_search_layout; workspace from
  * dtp_search_chain_workspace_size.  Asynchronous; invalid entries or loop
  * limits are reported through the workspace status word.

@@ -273,7 +273,7 @@ def down_score(act2, bn, T_total: int):
 
 
 def normalize_unit_mass(S):
-    """Exact integer unit-mass form of one affinity matrix (units of 2^-39)."""
+    """Exact integer unit-mass form of one affinity matrix (units of 2^-43)."""
     S = _c(S, np.float32)
     n = np.zeros(S.shape, dtype=np.int64)
     st = _load().oracle_normalize_unit_mass(_p(S, _f32p), S.size, _p(n, _i64p))
@@ -302,7 +302,7 @@ def chain_search(S_up, S_down, D: int, iters: int):
 
 
 def chain_score(S_up, S_down, h, nu) -> int:
-    """J of a layout over all layers (Eq. objective), in units of 2^-39."""
+    """J of a layout over all layers (Eq. objective), in units of 2^-43."""
     Su = _c(S_up, np.float32)
     L, G, N = Su.shape
     Sd = _c(S_down if L > 1 else np.zeros((1, G, N)), np.float32)

@@ -604,16 +604,18 @@ void oracle_down_score(const double* act2, const double* bn, int G, int N, int64
 /* Whole-model objective and optimiser (Sec. 3 "Objective", "Optimiser")     */
 /* ------------------------------------------------------------------------ */
 
-#define OR_NORM_BITS 39
-#define OR_NORM_PRE_BITS 24
+#define OR_NORM_BITS 43
+#define OR_NORM_PRE_BITS 40
 
 /*
  * Unit-mass normalisation (Sec. 3 "Objective": each matrix is normalised to
  * unit mass so every edge counts equally), in exact integers:
- *     q = floor(S * 2^(24-e)),  max(S) < 2^e          (q < 2^24)
- *     n = floor(q * 2^39 / sum(q))                     (sum(n) <= 2^39)
- * so n is the matrix's share of its own mass in units of 2^-39.  All-zero S
- * gives n = 0.  Returns -1 for a negative or non-finite entry.
+ *     q = floor(S * 2^(40-e)),  max(S) < 2^e          (q < 2^40)
+ *     n = floor(q * 2^43 / sum(q))                     (sum(n) <= 2^43)
+ * (the product q * 2^43 is formed in 128 bits), so n is the matrix's share of
+ * its own mass in units of 2^-43; a neuron's gain, summed over one up and one
+ * down matrix, stays below 2^44.  All-zero S gives n = 0.  Returns -1 for a
+ * negative or non-finite entry.
  */
 int oracle_normalize_unit_mass(const float* S, int64_t count, int64_t* n) {
     float smax = 0.0f;
@@ -634,7 +636,7 @@ int oracle_normalize_unit_mass(const float* S, int64_t count, int64_t* n) {
         total += (uint64_t)n[i];
     }
     for (int64_t i = 0; i < count; ++i)
-        n[i] = (int64_t)(((uint64_t)n[i] << OR_NORM_BITS) / total);
+        n[i] = (int64_t)((((unsigned __int128)(uint64_t)n[i]) << OR_NORM_BITS) / total);
     return OR_OK;
 }
 
@@ -649,7 +651,7 @@ int oracle_normalize_unit_mass(const float* S, int64_t count, int64_t* n) {
  * edge and nu_{i-1} for the down edge).  Given the other block, each step
  * maximises J exactly, so J never decreases.  Start: contiguous heads in every
  * layer.  Stop after `iters` or the first iteration without a strict increase.
- * J_q is J in units of 2^-39; *J = J_q / 2^39.
+ * J_q is J in units of 2^-43; *J = J_q / 2^43.
  */
 int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, int N, int D, int iters, int* h,
                         int* nu, int64_t* J_q, double* J, int* iters_done, int* all_unique) {
@@ -708,7 +710,7 @@ int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, in
     return OR_OK;
 }
 
-/* J of a given layout (both sums of Eq. objective), in units of 2^-39. */
+/* J of a given layout (both sums of Eq. objective), in units of 2^-43. */
 int64_t oracle_chain_score(const float* S_up, const float* S_down, int L, int G, int N, const int* h, const int* nu) {
     const int64_t GN = (int64_t)G * N;
     int64_t* n = (int64_t*)malloc(sizeof(int64_t) * (size_t)GN);

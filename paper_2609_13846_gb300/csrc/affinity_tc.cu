@@ -17,7 +17,10 @@
 // unit runs G+1 passes over d: pass 0 multiplies the X chunk, pass 1+h the C_h
 // chunk.  Units are dealt round-robin to a persistent grid in
 // token-chunk-major order, so the CTAs in flight share a handful of token
-// chunks in L2 while all weights stay L2-resident.  The units left over after
+// chunks in L2 while all weights stay L2-resident.  When the weights do not
+// fit in L2, token chunks are taken in groups and each neuron tile meets the
+// group's chunks back to back, so the units in flight share fewer weight
+// tiles.  The units left over after
 // the last full round are split by heads over several CTAs (each recomputes
 // the unit's X pass), so the final round keeps most SMs busy.
 //
@@ -82,6 +85,7 @@ struct Params {
     int full_rounds;  // rounds in which every CTA takes one whole unit
     int split;        // head groups per left-over unit
     int tail_items;   // left-over units * split (<= grid)
+    int cg;           // token chunks per group of the unit order (1 = chunk-major)
     int64_t T;        // tokens
     float* partial;   // [units][G][128]
     const float* rms; // [T] rms of the next layer's pre-norm input, or null
@@ -94,6 +98,17 @@ struct Item {
     int64_t unit;
     int h0, h1;
 };
+
+// Unit u in the processing order -> (token chunk c, neuron tile j).
+__device__ __forceinline__ void unit_coords(const Params& p, int64_t u, int& c, int& j) {
+    const int64_t per_group = static_cast<int64_t>(p.cg) * p.NT;
+    const int64_t grp = u / per_group;
+    const int64_t r = u - grp * per_group;
+    const int c0 = static_cast<int>(grp) * p.cg;
+    const int cn = p.TC - c0 < p.cg ? p.TC - c0 : p.cg;   // chunks in this (possibly last) group
+    j = static_cast<int>(r / cn);
+    c = c0 + static_cast<int>(r % cn);
+}
 
 __device__ __forceinline__ bool get_item(const Params& p, int i, Item& it) {
     if (i < p.full_rounds) {
@@ -192,8 +207,8 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
             bool ok = true;
             Item it;
             for (int i = 0; ok && get_item(p, i, it); ++i) {
-                const int c = static_cast<int>(it.unit / p.NT);
-                const int j = static_cast<int>(it.unit % p.NT);
+                int c, j;
+                unit_coords(p, it.unit, c, j);
                 const int passes = 1 + it.h1 - it.h0;
                 for (int pass = 0; ok && pass < passes; ++pass) {
                     for (int kb = 0; kb < p.KB; ++kb) {
@@ -308,7 +323,10 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
         };
         Item it;
         for (int i = 0; ok && get_item(p, i, it); ++i) {
-            float* out = p.partial + (it.unit * p.G + it.h0) * static_cast<int64_t>(BNEU);
+            int uc, uj;
+            unit_coords(p, it.unit, uc, uj);
+            const int64_t slot_unit = static_cast<int64_t>(uc) * p.NT + uj;   // partial slot: (chunk, tile)
+            float* out = p.partial + (slot_unit * p.G + it.h0) * static_cast<int64_t>(BNEU);
             const int passes = 1 + it.h1 - it.h0;
             for (int pass = 0; pass < passes; ++pass, ++pass_count) {
                 const uint32_t buf = pass_count & 1u;
@@ -321,7 +339,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                     const bool want_act = p.rms != nullptr && it.h0 == 0;
                     float ir2 = 0.0f;
                     if (want_act) {
-                        const int64_t tok = (it.unit / p.NT) * BT + quad * 32 + lane;
+                        const int64_t tok = static_cast<int64_t>(uc) * BT + quad * 32 + lane;
                         if (tok < p.T) {
                             const float r = p.rms[tok];
                             ir2 = 1.0f / (r * r);
@@ -350,7 +368,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                         if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
                         continue;
                     }
-                    if (!reduce_store(asum, p.partial_act + it.unit * BNEU + half * 64, buf)) { ok = false; break; }
+                    if (!reduce_store(asum, p.partial_act + slot_unit * BNEU + half * 64, buf)) { ok = false; break; }
                     continue;
                 }
                 // head pass: column sums of Delta^2 over this warp's 32 tokens
@@ -493,12 +511,20 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
                                                      align_up(workspace_bytes(T, d, G, N), 256))
                           : nullptr;
 
-    int dev = 0, sms = 0;
+    int dev = 0, sms = 0, l2 = 0;
     DTP_CUDA_TRY(cudaGetDevice(&dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    DTP_CUDA_TRY(cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev));
     DTP_CUDA_TRY(cudaFuncSetAttribute(affinity_fo_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       static_cast<int>(kSmemBytes)));
     const int grid = static_cast<int>(p.units < sms ? p.units : sms);
+    // chunk grouping: keep the weight tiles of the units in flight within a third of L2
+    {
+        const double tile_bytes = 2.0 * BNEU * d * 2.0;
+        p.cg = 1;
+        if (static_cast<double>(p.NT) * tile_bytes > l2 / 2.0)
+            while (p.cg < 64 && p.cg < p.TC && (static_cast<double>(grid) / p.cg) * tile_bytes > l2 / 3.0) p.cg *= 2;
+    }
     p.full_rounds = static_cast<int>(p.units / grid);
     const int left = static_cast<int>(p.units - static_cast<int64_t>(p.full_rounds) * grid);
     p.split = left > 0 ? (grid / left < G ? grid / left : G) : 1;

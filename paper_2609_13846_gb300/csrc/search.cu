@@ -14,7 +14,8 @@
 //   D == 2  device 0 takes the N/2 largest M[k,0]-M[k,1], lower index first on
 //           ties: one block-wide radix selection of packed (difference, index)
 //           keys.
-//   D >  2  (a) device prices pi from a few Gauss-Seidel sweeps, each price set
+//   D >  2  (a) device prices pi from Gauss-Seidel sweeps (until the excess
+//           over N/D is at most 2D neurons, at most kMaxSweeps), each price set
 //           by a radix selection so that about N/D neurons prefer its device;
 //           (b) every neuron to its best device at those prices -- optimal for
 //           the resulting device counts by complementary slackness;
@@ -45,6 +46,7 @@ constexpr int kFixedBits = 40;
 constexpr int kIdxBits = 18;                       // N <= 2^18
 constexpr int64_t kValBias = int64_t(1) << 45;     // |gain| < 2^44 (H_kv <= 16): fits the 46-bit field
 constexpr int64_t kNegInf = INT64_MIN / 4;
+constexpr int kMaxSweeps = 16;                      // price sweeps before the exact repair
 constexpr size_t kSmemBudget = 220 * 1024;         // dynamic smem for M, nu and (if it fits) A
 
 struct Shared {
@@ -333,7 +335,7 @@ template <int DT>
 __device__ void neuron_step_general(const Layer& L, Shared& sh) {
     const int N = L.N, D = L.D, cap = L.cap;
     // (a) price sweeps
-    for (int sweep = 0; sweep < 3; ++sweep) {
+    for (int sweep = 0; sweep < kMaxSweeps; ++sweep) {
         if (threadIdx.x < DMAX) sh.count[threadIdx.x] = 0;
         __syncthreads();
         for (int k = threadIdx.x; k < N; k += kThreads) atomicAdd(&sh.count[best_device<DT>(L, sh, k)], 1);
@@ -678,7 +680,8 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
 // ------------------------------------------------------- whole-model search --
 //
 // Eq. objective with both sums: J = sum_i up_i + sum_{i<L-1} down_i, each matrix
-// in its exact unit-mass form n = floor(floor(S 2^(24-e)) 2^39 / total).  One
+// in its exact unit-mass form n = floor(q 2^43 / total), q = floor(S 2^(40-e)),
+// the product taken in 128 bits.  One
 // iteration = every layer's neuron step given all head partitions (gain from
 // h_i for the up edge and h_{i+1} for the down edge), then every layer's head
 // step given all neuron assignments (column sums over nu_i for the up edge and
@@ -687,8 +690,8 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
 // flag stops later iterations after the first one without a strict increase,
 // so the host never waits.
 
-constexpr int kNormBits = 39;
-constexpr int kNormPreBits = 24;
+constexpr int kNormBits = 43;   // gains (one up + one down matrix) stay below 2^44
+constexpr int kNormPreBits = 40;
 
 struct ChainState {
     int done;
@@ -739,7 +742,7 @@ chain_normalize_kernel(const float* __restrict__ S_up, const float* __restrict__
     const uint64_t total = static_cast<uint64_t>(block_sum_i64(part, sh));
     for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
         const uint64_t q = static_cast<uint64_t>(quantize_bits(src[i], e, kNormPreBits));
-        dst[i] = total ? static_cast<int64_t>((q << kNormBits) / total) : 0;
+        dst[i] = total ? static_cast<int64_t>((static_cast<unsigned __int128>(q) << kNormBits) / total) : 0;
     }
 }
 

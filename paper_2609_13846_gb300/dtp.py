@@ -316,7 +316,7 @@ def search_chain(S_up: torch.Tensor, S_down: torch.Tensor | None, D: int, iters:
 
     S_up [L, H_kv, N], S_down [L-1, H_kv, N] (None when L == 1), fp32 CUDA.
     Returns device tensors: h [L,H_kv] int32, nu [L,N] int32, J_q int64 (units
-    of 2^-39), J float64, iters_done int32.  Asynchronous unless ``check``.
+    of 2^-43), J float64, iters_done int32.  Asynchronous unless ``check``.
     """
     if S_up.dtype != torch.float32 or not S_up.is_cuda or not S_up.is_contiguous():
         raise ValueError("S_up must be a contiguous fp32 CUDA tensor [L, H_kv, N]")

@@ -48,6 +48,7 @@ class Workload:
     seed: int = 0
     outliers: bool = True
     iters: int = 10
+    qkv_rows: int = 512   # next layer's q/k/v rows per KV group: (query heads per group + 2) * head_dim
 
     def layer_seed(self, layer: int) -> int:
         """Seed of layer ``layer``: the workload seed plus the layer index."""
@@ -57,15 +58,15 @@ class Workload:
 # The five calibration workloads.  FLOP per token of the affinity pass is
 # 2*d*2N*(G+1).
 WORKLOADS = {
-    "tiny": Workload("tiny", d=64, G=2, N=128, T=256, D=(2,), dtype="f32", seed=0, outliers=False),
+    "tiny": Workload("tiny", d=64, G=2, N=128, T=256, D=(2,), dtype="f32", seed=0, outliers=False, qkv_rows=64),
     "qwen3_0.6b_layer": Workload("qwen3_0.6b_layer", d=1024, G=8, N=3072, T=16384, D=(2,),
                                  dtype="bf16", seed=1),
     "qwen3_0.6b_model": Workload("qwen3_0.6b_model", d=1024, G=8, N=3072, T=65536, D=(2, 4),
                                  dtype="bf16", layers=28, seed=100),
     "danube3_500m_model": Workload("danube3_500m_model", d=1536, G=8, N=4096, T=65536, D=(4,),
-                                   dtype="bf16", layers=16, seed=200),
+                                   dtype="bf16", layers=16, seed=200, qkv_rows=384),
     "llama3.1_8b_layer": Workload("llama3.1_8b_layer", d=4096, G=8, N=14336, T=32768, D=(4, 8),
-                                  dtype="bf16", seed=3),
+                                  dtype="bf16", seed=3, qkv_rows=768),
 }
 
 

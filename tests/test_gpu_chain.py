@@ -1,7 +1,7 @@
 """GPU parity of the whole-model optimiser (Sec. 3, Eq. objective with both edges) against the oracle.
 
 Both sides get the same fp32 S_up and S_down; the contract is bit-exact on
-every layer's head partition and neuron assignment, on J in units of 2^-39
+every layer's head partition and neuron assignment, on J in units of 2^-43
 and on the iteration count.
 """
 import numpy as np

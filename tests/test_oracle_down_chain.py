@@ -91,9 +91,9 @@ def test_unit_mass_normalisation():
     S = synth.make_affinity_matrix(4, 50, seed=3).numpy()
     n = oracle.normalize_unit_mass(S)
     total = int(n.sum())
-    assert total <= 2 ** 39 and total >= 2 ** 39 - 2 * S.size
-    ratio = n / 2.0 ** 39
-    np.testing.assert_allclose(ratio, S / S.sum(), atol=2.0 ** -22 * 4)   # 24-bit pre-quantisation
+    assert total <= 2 ** 43 and total >= 2 ** 43 - 2 * S.size
+    ratio = n / 2.0 ** 43
+    np.testing.assert_allclose(ratio, S / S.sum(), rtol=1e-6, atol=2.0 ** -36)   # 40-bit pre-quantisation
     for k in (-5, 7):
         np.testing.assert_array_equal(oracle.normalize_unit_mass(S * np.float32(2.0 ** k)), n)
     assert not oracle.normalize_unit_mass(np.zeros((2, 3), np.float32)).any()
@@ -163,6 +163,6 @@ def test_random_layout_expectation_matches_paper():
         for _ in range(60):
             h = np.stack([rng.permutation(np.repeat(np.arange(4), 2)) for _ in range(layers)]).astype(np.int32)
             nu = np.stack([rng.permutation(np.repeat(np.arange(4), 16)) for _ in range(layers)]).astype(np.int32)
-            vals.append(oracle.chain_score(Su, Sd, h, nu) / 2.0 ** 39)
+            vals.append(oracle.chain_score(Su, Sd, h, nu) / 2.0 ** 43)
         mean, sem = float(np.mean(vals)), float(np.std(vals) / np.sqrt(len(vals)))
         assert abs(mean - gold[key]["value"]) < 4 * sem + 0.05
