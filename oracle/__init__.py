@@ -88,8 +88,15 @@ def _load():
     lib.oracle_chain_search.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                         ctypes.c_int, _i32p, _i32p, _i64p, _f64p, _i32p, _i32p]
     lib.oracle_chain_search.restype = ctypes.c_int
+    lib.oracle_chain_search_ex.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                           ctypes.c_int, ctypes.c_char_p, ctypes.c_char_p, ctypes.c_int, _i32p, _i32p,
+                                           _i64p, _f64p, _i32p, _i32p]
+    lib.oracle_chain_search_ex.restype = ctypes.c_int
     lib.oracle_chain_score.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p]
     lib.oracle_chain_score.restype = ctypes.c_int64
+    lib.oracle_chain_edge_scores.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p,
+                                             _i64p]
+    lib.oracle_chain_edge_scores.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -282,8 +289,12 @@ def normalize_unit_mass(S):
     return n
 
 
-def chain_search(S_up, S_down, D: int, iters: int):
-    """Coordinate ascent on the whole-model objective (both edges): dict(h, nu, J_q, J, iters_done, unique)."""
+def chain_search(S_up, S_down, D: int, iters: int, move_heads=None, move_neurons=None, minimize=False):
+    """Coordinate ascent on the whole-model objective (both edges): dict(h, nu, J_q, J, iters_done, unique).
+
+    move_heads / move_neurons: per-layer 0/1 (None = every layer moves); minimize: the
+    anti-optimised layout (Sec. 3 'Optimiser', Table 4 ablations).
+    """
     Su = _c(S_up, np.float32)
     L, G, N = Su.shape
     Sd = _c(S_down if L > 1 else np.zeros((1, G, N)), np.float32)
@@ -294,8 +305,11 @@ def chain_search(S_up, S_down, D: int, iters: int):
     j = ctypes.c_double(0.0)
     it = ctypes.c_int(0)
     uq = ctypes.c_int(0)
-    st = _load().oracle_chain_search(_p(Su, _f32p), _p(Sd, _f32p), L, G, N, D, iters, _p(h, _i32p), _p(nu, _i32p),
-                                     ctypes.byref(jq), ctypes.byref(j), ctypes.byref(it), ctypes.byref(uq))
+    mh = None if move_heads is None else bytes(np.asarray(move_heads, dtype=np.uint8).tolist())
+    mn = None if move_neurons is None else bytes(np.asarray(move_neurons, dtype=np.uint8).tolist())
+    st = _load().oracle_chain_search_ex(_p(Su, _f32p), _p(Sd, _f32p), L, G, N, D, iters, mh, mn, int(minimize),
+                                        _p(h, _i32p), _p(nu, _i32p), ctypes.byref(jq), ctypes.byref(j),
+                                        ctypes.byref(it), ctypes.byref(uq))
     if st != 0:
         raise ValueError(f"oracle_chain_search: status {st}")
     return dict(h=h, nu=nu, J_q=int(jq.value), J=float(j.value), iters_done=int(it.value), unique=bool(uq.value))
@@ -308,3 +322,16 @@ def chain_score(S_up, S_down, h, nu) -> int:
     Sd = _c(S_down if L > 1 else np.zeros((1, G, N)), np.float32)
     return int(_load().oracle_chain_score(_p(Su, _f32p), _p(Sd, _f32p), L, G, N, _p(_c(h, np.int32), _i32p),
                                           _p(_c(nu, np.int32), _i32p)))
+
+
+def chain_edge_scores(S_up, S_down, h, nu) -> np.ndarray:
+    """Co-located mass per edge [2L-1] (up_0, down_0, up_1, ..., up_{L-1}), units of 2^-43 of each edge."""
+    Su = _c(S_up, np.float32)
+    L, G, N = Su.shape
+    Sd = _c(S_down if L > 1 else np.zeros((1, G, N)), np.float32)
+    out = np.zeros(2 * L - 1, np.int64)
+    bad = _load().oracle_chain_edge_scores(_p(Su, _f32p), _p(Sd, _f32p), L, G, N, _p(_c(h, np.int32), _i32p),
+                                           _p(_c(nu, np.int32), _i32p), _p(out, _i64p))
+    if bad:
+        raise ValueError("negative or non-finite affinity entry")
+    return out

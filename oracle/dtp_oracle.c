@@ -649,15 +649,22 @@ int oracle_normalize_unit_mass(const float* S, int64_t count, int64_t* n) {
  * One iteration: every layer's neuron step given all h (gain M_kl of Sec. 3),
  * then every layer's head step given all nu (column sums over nu_i for the up
  * edge and nu_{i-1} for the down edge).  Given the other block, each step
- * maximises J exactly, so J never decreases.  Start: contiguous heads in every
- * layer.  Stop after `iters` or the first iteration without a strict increase.
- * J_q is J in units of 2^-43; *J = J_q / 2^43.
+ * maximises J exactly, so J never decreases.  Start: contiguous heads and
+ * neurons in every layer.  Stop after `iters` or the first iteration (after
+ * the first) without a strict increase.  J_q is J in units of 2^-43.
+ *
+ * Ablations (Sec. 3 "Optimiser", Table 4): move_heads[i] == 0 keeps layer i's
+ * heads contiguous, move_neurons[i] == 0 its neurons (NULL = every layer
+ * moves); minimize != 0 minimises J instead (the anti-optimised layout) by
+ * maximising -J with the same exact steps.
  */
-int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, int N, int D, int iters, int* h,
-                        int* nu, int64_t* J_q, double* J, int* iters_done, int* all_unique) {
+int oracle_chain_search_ex(const float* S_up, const float* S_down, int L, int G, int N, int D, int iters,
+                           const unsigned char* move_heads, const unsigned char* move_neurons, int minimize,
+                           int* h, int* nu, int64_t* J_q, double* J, int* iters_done, int* all_unique) {
     if (L < 1 || D < 2 || D > OR_DMAX || G <= 0 || G % D || G > OR_GMAX || N <= 0 || N % D || iters < 1)
         return OR_ERR_ARG;
     const int64_t GN = (int64_t)G * N;
+    const int64_t sign = minimize ? -1 : 1;
     int64_t* nU = (int64_t*)malloc(sizeof(int64_t) * (size_t)(L * GN));
     int64_t* nD = (int64_t*)malloc(sizeof(int64_t) * (size_t)((L > 1 ? L - 1 : 1) * GN));
     int64_t* M = (int64_t*)malloc(sizeof(int64_t) * (size_t)N * D);
@@ -665,18 +672,21 @@ int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, in
     for (int i = 0; i < L && status == OR_OK; ++i) status = oracle_normalize_unit_mass(S_up + i * GN, GN, nU + i * GN);
     for (int i = 0; i + 1 < L && status == OR_OK; ++i)
         status = oracle_normalize_unit_mass(S_down + i * GN, GN, nD + i * GN);
-    for (int i = 0; i < L; ++i)
+    for (int i = 0; i < L; ++i) {
         for (int g = 0; g < G; ++g) h[i * G + g] = (g * D) / G;
-    int64_t prev = -1, total = 0;
+        for (int k = 0; k < N; ++k) nu[(int64_t)i * N + k] = (int)(((int64_t)k * D) / N);
+    }
+    int64_t prev = 0, total = 0;
     int done = 0, uniq_all = 1;
     for (int it = 0; it < iters && status == OR_OK; ++it) {
         for (int i = 0; i < L && status == OR_OK; ++i) {
-            /* M[k,l] = up gain from h_i + down gain from h_{i+1} */
+            if (move_neurons && !move_neurons[i]) continue;
+            /* M[k,l] = sign * (up gain from h_i + down gain from h_{i+1}) */
             memset(M, 0, sizeof(int64_t) * (size_t)N * D);
             for (int g = 0; g < G; ++g)
                 for (int k = 0; k < N; ++k) {
-                    M[(int64_t)k * D + h[i * G + g]] += nU[i * GN + (int64_t)g * N + k];
-                    if (i + 1 < L) M[(int64_t)k * D + h[(i + 1) * G + g]] += nD[i * GN + (int64_t)g * N + k];
+                    M[(int64_t)k * D + h[i * G + g]] += sign * nU[i * GN + (int64_t)g * N + k];
+                    if (i + 1 < L) M[(int64_t)k * D + h[(i + 1) * G + g]] += sign * nD[i * GN + (int64_t)g * N + k];
                 }
             int uniq = 1;
             status = neuron_step_from_gain(M, N, D, nu + (int64_t)i * N, &uniq, 0);
@@ -685,29 +695,39 @@ int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, in
         if (status != OR_OK) break;
         total = 0;
         for (int i = 0; i < L; ++i) {
-            /* B[g,l] = up mass of g on device l under nu_i + down mass into g under nu_{i-1} */
+            /* B[g,l] = sign * (up mass of g on device l under nu_i + down mass into g under nu_{i-1}) */
             int64_t B[OR_GMAX * OR_DMAX];
             memset(B, 0, sizeof(B));
             for (int g = 0; g < G; ++g)
                 for (int k = 0; k < N; ++k) {
-                    B[g * D + nu[(int64_t)i * N + k]] += nU[i * GN + (int64_t)g * N + k];
-                    if (i > 0) B[g * D + nu[(int64_t)(i - 1) * N + k]] += nD[(i - 1) * GN + (int64_t)g * N + k];
+                    B[g * D + nu[(int64_t)i * N + k]] += sign * nU[i * GN + (int64_t)g * N + k];
+                    if (i > 0) B[g * D + nu[(int64_t)(i - 1) * N + k]] += sign * nD[(i - 1) * GN + (int64_t)g * N + k];
                 }
             int64_t sc = 0;
-            head_step_from_sums(B, G, D, h + i * G, &sc);
+            if (move_heads && !move_heads[i]) {
+                for (int g = 0; g < G; ++g) sc += B[g * D + h[i * G + g]];
+            } else {
+                head_step_from_sums(B, G, D, h + i * G, &sc);
+            }
             total += sc;
         }
         done = it + 1;
-        if (total <= prev) break;
+        if (it > 0 && total <= prev) break;
         prev = total;
     }
     free(nU); free(nD); free(M);
     if (status != OR_OK) return status;
-    *J_q = total;
-    *J = ldexp((double)total, -OR_NORM_BITS);
+    *J_q = sign * total;
+    *J = ldexp((double)(sign * total), -OR_NORM_BITS);
     *iters_done = done;
     if (all_unique) *all_unique = uniq_all;
     return OR_OK;
+}
+
+int oracle_chain_search(const float* S_up, const float* S_down, int L, int G, int N, int D, int iters, int* h,
+                        int* nu, int64_t* J_q, double* J, int* iters_done, int* all_unique) {
+    return oracle_chain_search_ex(S_up, S_down, L, G, N, D, iters, NULL, NULL, 0, h, nu, J_q, J, iters_done,
+                                  all_unique);
 }
 
 /* J of a given layout (both sums of Eq. objective), in units of 2^-43. */
@@ -729,6 +749,40 @@ int64_t oracle_chain_score(const float* S_up, const float* S_down, int L, int G,
     }
     free(n);
     return J;
+}
+
+/*
+ * Per-edge co-located mass of a layout, in units of 2^-43 of each edge's own
+ * unit mass: edge[2i] = up_i, edge[2i+1] = down_i (i < L-1); 2L-1 entries.
+ * up_i / 2^43 is the co-located fraction of layer i's up edge (0.25 expected
+ * for a random layout at four devices).  Returns the number of invalid
+ * matrices (0 on success).
+ */
+int oracle_chain_edge_scores(const float* S_up, const float* S_down, int L, int G, int N, const int* h, const int* nu,
+                             int64_t* edge) {
+    const int64_t GN = (int64_t)G * N;
+    int64_t* n = (int64_t*)malloc(sizeof(int64_t) * (size_t)GN);
+    int bad = 0;
+    for (int i = 0; i < L; ++i) {
+        int64_t e = 0;
+        if (oracle_normalize_unit_mass(S_up + i * GN, GN, n) != OR_OK) ++bad;
+        else
+            for (int g = 0; g < G; ++g)
+                for (int k = 0; k < N; ++k)
+                    if (h[i * G + g] == nu[(int64_t)i * N + k]) e += n[(int64_t)g * N + k];
+        edge[2 * i] = e;
+        if (i + 1 < L) {
+            e = 0;
+            if (oracle_normalize_unit_mass(S_down + i * GN, GN, n) != OR_OK) ++bad;
+            else
+                for (int g = 0; g < G; ++g)
+                    for (int k = 0; k < N; ++k)
+                        if (nu[(int64_t)i * N + k] == h[(i + 1) * G + g]) e += n[(int64_t)g * N + k];
+            edge[2 * i + 1] = e;
+        }
+    }
+    free(n);
+    return bad;
 }
 
 /* ------------------------------------------------------------------------ */

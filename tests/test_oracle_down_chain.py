@@ -166,3 +166,126 @@ def test_random_layout_expectation_matches_paper():
             vals.append(oracle.chain_score(Su, Sd, h, nu) / 2.0 ** 43)
         mean, sem = float(np.mean(vals)), float(np.std(vals) / np.sqrt(len(vals)))
         assert abs(mean - gold[key]["value"]) < 4 * sem + 0.05
+
+
+# ------------------------------------------------------------- ablations ----
+# Sec. 3 "Optimiser": restricting which layers move, freezing heads or
+# neurons, or minimising J gives the ablation layouts of Table 4.
+
+from paper_2609_13846_gb300 import ablation  # noqa: E402
+
+
+def _contiguous(L, G, N, D):
+    h = np.stack([np.array([(g * D) // G for g in range(G)], np.int32)] * L)
+    nu = np.stack([np.array([(k * D) // N for k in range(N)], np.int32)] * L)
+    return h, nu
+
+
+@pytest.mark.parametrize("L,seed", [(2, 3), (3, 4)])
+def test_neurons_only_is_the_exact_optimum_over_neurons(L, seed):
+    """Heads frozen contiguous: the neuron steps of different layers are independent given h, so
+    one sweep reaches the global optimum over every nu; brute force over all of them."""
+    G, N, D = 2, 4, 2
+    Su, Sd = _random_model(L, G, N, seed)
+    h0, nu0 = _contiguous(L, G, N, D)
+    nus = list(_balanced(N, D))
+    best = max(oracle.chain_score(Su, Sd, h0, np.stack(nu)) for nu in itertools.product(nus, repeat=L))
+    res = oracle.chain_search(Su, Sd, D, 10, move_heads=np.zeros(L), move_neurons=np.ones(L))
+    np.testing.assert_array_equal(res["h"], h0)
+    assert res["J_q"] == best == oracle.chain_score(Su, Sd, res["h"], res["nu"])
+    worst = min(oracle.chain_score(Su, Sd, h0, np.stack(nu)) for nu in itertools.product(nus, repeat=L))
+    anti = oracle.chain_search(Su, Sd, D, 10, move_heads=np.zeros(L), minimize=True)
+    assert anti["J_q"] == worst == oracle.chain_score(Su, Sd, anti["h"], anti["nu"])
+
+
+@pytest.mark.parametrize("L,seed", [(2, 5), (3, 6)])
+def test_heads_only_is_the_exact_optimum_over_heads(L, seed):
+    G, N, D = 4, 4, 2
+    Su, Sd = _random_model(L, G, N, seed)
+    h0, nu0 = _contiguous(L, G, N, D)
+    hs = list(_balanced(G, D))
+    best = max(oracle.chain_score(Su, Sd, np.stack(h), nu0) for h in itertools.product(hs, repeat=L))
+    res = oracle.chain_search(Su, Sd, D, 10, move_heads=np.ones(L), move_neurons=np.zeros(L))
+    np.testing.assert_array_equal(res["nu"], nu0)
+    assert res["J_q"] == best
+    worst = min(oracle.chain_score(Su, Sd, np.stack(h), nu0) for h in itertools.product(hs, repeat=L))
+    anti = oracle.chain_search(Su, Sd, D, 10, move_neurons=np.zeros(L), minimize=True)
+    assert anti["J_q"] == worst
+
+
+@pytest.mark.parametrize("L,seed", [(2, 7), (3, 8)])
+def test_anti_optimised_against_brute_force(L, seed):
+    """Minimising J: the result's J is its layout's J, at or above the global minimum, and the
+    first sweep's neuron and head steps are exact minimisers."""
+    G, N, D = 2, 4, 2
+    Su, Sd = _random_model(L, G, N, seed)
+    hs, nus = list(_balanced(G, D)), list(_balanced(N, D))
+    worst = min(oracle.chain_score(Su, Sd, np.stack(h), np.stack(nu))
+                for h in itertools.product(hs, repeat=L) for nu in itertools.product(nus, repeat=L))
+    res = oracle.chain_search(Su, Sd, D, 10, minimize=True)
+    assert res["J_q"] == oracle.chain_score(Su, Sd, res["h"], res["nu"]) >= worst
+    one = oracle.chain_search(Su, Sd, D, 1, minimize=True)
+    h0, _ = _contiguous(L, G, N, D)
+    assert oracle.chain_score(Su, Sd, h0, one["nu"]) == min(
+        oracle.chain_score(Su, Sd, h0, np.stack(nu)) for nu in itertools.product(nus, repeat=L))
+    assert one["J_q"] == min(oracle.chain_score(Su, Sd, np.stack(h), one["nu"]) for h in itertools.product(hs, repeat=L))
+
+
+def test_layer_subset_keeps_other_layers_contiguous():
+    L, G, N, D = 6, 8, 64, 4
+    Su, Sd = _random_model(L, G, N, seed=12)
+    h0, nu0 = _contiguous(L, G, N, D)
+    mh, mn, mini = ablation.ablation_masks(L, "layers2")
+    assert list(np.flatnonzero(mh)) == [0, 3] and not mini
+    res = oracle.chain_search(Su, Sd, D, 10, move_heads=mh, move_neurons=mn)
+    for i in range(L):
+        if not mh[i]:
+            np.testing.assert_array_equal(res["h"][i], h0[i])
+            np.testing.assert_array_equal(res["nu"][i], nu0[i])
+    assert res["J_q"] == oracle.chain_score(Su, Sd, res["h"], res["nu"])
+    assert res["J_q"] >= oracle.chain_score(Su, Sd, h0, nu0)
+    frozen = oracle.chain_search(Su, Sd, D, 10, move_heads=np.zeros(L), move_neurons=np.zeros(L))
+    assert frozen["J_q"] == oracle.chain_score(Su, Sd, h0, nu0) and frozen["iters_done"] == 2
+
+
+def test_ablation_ordering_invariants():
+    """anti <= contiguous <= neurons-only <= optimised (the full ascent's first neuron sweep is
+    the neurons-only layout, and every later step can only raise J); anti < random mean < optimised."""
+    L, G, N, D = 8, 8, 128, 4
+    Su, Sd = _random_model(L, G, N, seed=21)
+    h0, nu0 = _contiguous(L, G, N, D)
+    J = {k: oracle.chain_search(Su, Sd, D, 10, *[None if m is None else m for m in ablation.ablation_masks(L, k)[:2]],
+                                minimize=ablation.ablation_masks(L, k)[2])["J_q"]
+         for k in ("optimised", "anti", "heads_only", "neurons_only", "layers4")}
+    Jc = oracle.chain_score(Su, Sd, h0, nu0)
+    assert J["anti"] <= Jc <= J["neurons_only"] <= J["optimised"]
+    assert Jc <= J["heads_only"] and Jc <= J["layers4"]
+    rnd = np.mean([oracle.chain_score(Su, Sd, *ablation.random_layout(L, G, N, D, 1000 + s)) for s in range(8)])
+    assert J["anti"] < rnd < J["optimised"]
+
+
+def test_edge_scores_sum_to_the_objective_and_give_fractions():
+    L, G, N, D = 5, 8, 96, 4
+    Su, Sd = _random_model(L, G, N, seed=30)
+    h, nu = ablation.random_layout(L, G, N, D, 1001)
+    e = oracle.chain_edge_scores(Su, Sd, h, nu)
+    assert e.shape == (2 * L - 1,) and int(e.sum()) == oracle.chain_score(Su, Sd, h, nu)
+    # every layer on one device: each edge keeps all of its unit mass (up to the floor per entry)
+    h1, nu1 = np.zeros((L, G), np.int32), np.zeros((L, N), np.int32)
+    e1 = oracle.chain_edge_scores(Su, Sd, h1, nu1)
+    assert np.all(e1 <= 2 ** 43) and np.all(e1 >= 2 ** 43 - G * N)
+    # a layer whose heads and neurons sit on disjoint devices keeps none of its up edge
+    h2 = h1.copy(); h2[2] = 1
+    assert oracle.chain_edge_scores(Su, Sd, h2, nu1)[4] == 0
+
+
+def test_evenly_spaced_layers():
+    assert ablation.evenly_spaced_layers(28, 4) == [0, 7, 14, 21]
+    for L, n in ((28, 8), (28, 12), (16, 4), (16, 12), (5, 5)):
+        ls = ablation.evenly_spaced_layers(L, n)
+        assert ls[0] == 0 and len(set(ls)) == n and ls == sorted(ls) and ls[-1] < L
+    with pytest.raises(ValueError):
+        ablation.evenly_spaced_layers(4, 5)
+    h, nu = ablation.random_layout(3, 8, 64, 4, 1000)
+    assert all(np.bincount(r, minlength=4).tolist() == [2] * 4 for r in h)
+    assert all(np.bincount(r, minlength=4).tolist() == [16] * 4 for r in nu)
