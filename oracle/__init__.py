@@ -133,6 +133,29 @@ def affinity_fo(X, C, W_gate, W_up) -> np.ndarray:
     return A
 
 
+def affinity_fo_qheads(X, C_q, W_gate, W_up, q_per_group: int) -> np.ndarray:
+    """The first-order score per query head, summed over each KV group's query heads (Sec. 3).
+
+    C_q [H_q, T, d] holds each query head's own write p_h; row g of the result
+    is sum over h = g*q_per_group .. (g+1)*q_per_group - 1 of sum_t Delta_{t,h,k}^2
+    (a sum of per-head squares).  [H_q / q_per_group, N] fp64.
+    """
+    A = affinity_fo(X, C_q, W_gate, W_up)
+    H = A.shape[0]
+    if q_per_group < 1 or H % q_per_group:
+        raise ValueError("q_per_group must divide the number of query heads")
+    return A.reshape(H // q_per_group, q_per_group, -1).sum(axis=1)
+
+
+def affinity_add_qheads(C_q, W_gate, W_up, q_per_group: int) -> np.ndarray:
+    """The ADD score per query head, summed over each KV group's query heads (Sec. 3)."""
+    A = affinity_add(C_q, W_gate, W_up)
+    H = A.shape[0]
+    if q_per_group < 1 or H % q_per_group:
+        raise ValueError("q_per_group must divide the number of query heads")
+    return A.reshape(H // q_per_group, q_per_group, -1).sum(axis=1)
+
+
 def affinity_add(C, W_gate, W_up) -> np.ndarray:
     """ADD score before the mean: sum_t (p_h . w^g_k)^2 + (p_h . w^u_k)^2 (Sec. 3), fp64."""
     C = _c(C, np.float64)

@@ -223,3 +223,51 @@ def test_add_score_ignores_the_operating_point_and_fo_does_not():
     F1 = oracle.affinity_fo(X, C, Wg, Wu)
     F2 = oracle.affinity_fo(2.0 * X, C, Wg, Wu)
     assert np.max(np.abs(F1 - F2)) > 1e-3 * np.max(F1)
+
+
+# ------------------------------------------------ per-query-head scores ----
+# Sec. 3: the damage is taken per query head from that head's own write, and a
+# KV group's score is the sum over its query heads of E[Delta^2].
+
+def test_query_head_sum_with_one_head_per_group_is_plain_fo():
+    X, C, Wg, Wu = _tiny(seed=40, G=4)
+    np.testing.assert_array_equal(oracle.affinity_fo_qheads(X, C, Wg, Wu, 1), oracle.affinity_fo(X, C, Wg, Wu))
+    np.testing.assert_array_equal(oracle.affinity_add_qheads(C, Wg, Wu, 1), oracle.affinity_add(C, Wg, Wu))
+
+
+def test_query_head_sum_is_a_sum_of_squares_not_the_square_of_the_sum():
+    """Duplicated query heads (each group's heads all equal to c): Delta is linear in the write,
+    so the group's combined write q*c scores q^2 E[Delta_c^2] while the per-query-head sum is
+    q E[Delta_c^2]; the groups are consecutive heads."""
+    X, c, Wg, Wu = _tiny(seed=41, G=3)
+    for q in (2, 4):
+        Cq = np.repeat(c, q, axis=0)                      # heads g*q .. g*q+q-1 all equal c[g]
+        per_q = oracle.affinity_fo_qheads(X, Cq, Wg, Wu, q)
+        combined = oracle.affinity_fo(X, q * c, Wg, Wu)
+        np.testing.assert_allclose(per_q, combined / q, rtol=1e-12)
+        np.testing.assert_allclose(per_q, q * oracle.affinity_fo(X, c, Wg, Wu), rtol=1e-12)
+        np.testing.assert_allclose(oracle.affinity_add_qheads(Cq, Wg, Wu, q),
+                                   oracle.affinity_add(q * c, Wg, Wu) / q, rtol=1e-12)
+
+
+def test_query_head_sum_with_silent_heads_equals_group_write():
+    """A group whose other query heads write nothing: both readings agree."""
+    X, c, Wg, Wu = _tiny(seed=42, G=2)
+    Cq = np.zeros((6, *c.shape[1:]))
+    Cq[0], Cq[3] = c[0], c[1]                              # q = 3: one live head per group
+    np.testing.assert_allclose(oracle.affinity_fo_qheads(X, Cq, Wg, Wu, 3), oracle.affinity_fo(X, c, Wg, Wu),
+                               rtol=1e-13)
+
+
+def test_query_head_sum_against_finite_differences():
+    X, C, Wg, Wu = _tiny(seed=43, G=4, T=48)
+    g, u = X @ Wg.T, X @ Wu.T
+    eps = 1e-4
+    expect = np.zeros((2, Wg.shape[0]))
+    for h in range(4):
+        pg, pu = C[h] @ Wg.T, C[h] @ Wu.T
+        d = (_silu(g + eps * pg) * (u + eps * pu) - _silu(g - eps * pg) * (u - eps * pu)) / (2 * eps)
+        expect[h // 2] += (d ** 2).sum(axis=0)
+    np.testing.assert_allclose(oracle.affinity_fo_qheads(X, C, Wg, Wu, 2), expect, rtol=1e-6)
+    with pytest.raises(ValueError):
+        oracle.affinity_fo_qheads(X, C, Wg, Wu, 3)
