@@ -89,8 +89,8 @@ void oracle_affinity_fo(const double* X, const double* C, const double* Wg, cons
     for (int k = 0; k < N; ++k) {
         const double* wg = Wg + (int64_t)k * d;
         const double* wu = Wu + (int64_t)k * d;
-        double acc[OR_GMAX];
-        for (int h = 0; h < G; ++h) acc[h] = 0.0;
+        /* column k of A belongs to this iteration alone; any number of heads */
+        for (int h = 0; h < G; ++h) A[(int64_t)h * N + k] = 0.0;
         for (int64_t t = 0; t < T; ++t) {
             const double* x = X + t * d;
             double g = dot(x, wg, d);
@@ -103,10 +103,9 @@ void oracle_affinity_fo(const double* X, const double* C, const double* Wg, cons
                 double pg = dot(p, wg, d);
                 double pu = dot(p, wu, d);
                 double delta = dsilu * u * pg + silu * pu;
-                acc[h] += delta * delta;
+                A[(int64_t)h * N + k] += delta * delta;
             }
         }
-        for (int h = 0; h < G; ++h) A[(int64_t)h * N + k] = acc[h];
     }
 }
 

@@ -271,3 +271,12 @@ def test_query_head_sum_against_finite_differences():
     np.testing.assert_allclose(oracle.affinity_fo_qheads(X, C, Wg, Wu, 2), expect, rtol=1e-6)
     with pytest.raises(ValueError):
         oracle.affinity_fo_qheads(X, C, Wg, Wu, 3)
+
+
+def test_more_than_sixteen_heads_equal_split_calls():
+    """32 query heads (Llama-3.1-8B: 4 per KV group) in one call equal two 16-head calls."""
+    X, C, Wg, Wu = _tiny(seed=44, G=32, T=24)
+    A = oracle.affinity_fo(X, C, Wg, Wu)
+    np.testing.assert_array_equal(A, np.concatenate([oracle.affinity_fo(X, C[:16], Wg, Wu),
+                                                     oracle.affinity_fo(X, C[16:], Wg, Wu)]))
+    assert oracle.affinity_fo_qheads(X, C, Wg, Wu, 4).shape == (8, Wg.shape[0])
