@@ -188,6 +188,57 @@ def cpu_baseline(w, A_gpu, budget_s: float):
             "search_ms": 1e3 * t_search}
 
 
+def layout_suite(args, w, S_up, S_down, S_add, stream):
+    """The layouts of Table 4 on this model's affinities at one device count: the optimised layout,
+    the ablations (anti-optimised, heads only, neurons only, 4/8/12 evenly spaced layers), the ADD-score
+    layout when S_add is given (searched on the ADD up edge, scored under the first-order objective),
+    and eight random layouts (seeds 1000-1007) scored with chain_score.  Returns per-layout J and the
+    device time of the whole suite."""
+    from paper_2609_13846_gb300 import ablation, dtp
+    Lyr, G, N = S_up.shape
+    D = 4 if 4 in w.D else w.D[0]
+    Sd = S_down if Lyr > 1 else None
+    kinds = ["optimised", "anti", "heads_only", "neurons_only"] + \
+        [f"layers{n}" for n in (4, 8, 12) if n < Lyr]
+    masks = {k: ablation.ablation_masks(Lyr, k) for k in kinds}
+    dev_masks = {k: (None if mh is None else torch.as_tensor(mh, device=S_up.device),
+                     None if mn is None else torch.as_tensor(mn, device=S_up.device), mini)
+                 for k, (mh, mn, mini) in masks.items()}
+    rand = [tuple(torch.as_tensor(a, device=S_up.device) for a in ablation.random_layout(Lyr, G, N, D, 1000 + s))
+            for s in range(8)]
+    ws = torch.empty(dtp.search_chain_workspace_size(Lyr, G, N, D), dtype=torch.uint8, device=S_up.device)
+
+    def run(check):
+        out = {}
+        for k, (mh, mn, mini) in dev_masks.items():
+            out[k] = dtp.search_chain(S_up, Sd, D, w.iters, workspace=ws, check=check, move_heads=mh,
+                                      move_neurons=mn, minimize=mini)
+            out[k] = {"J": out[k]["J"].clone(), "iters": out[k]["iters_done"].clone()}
+        if S_add is not None:
+            r = dtp.search_chain(S_add, Sd, D, w.iters, workspace=ws, check=check)
+            sc = dtp.chain_score(S_up, Sd, r["h"], r["nu"], D, workspace=ws, check=check)
+            out["add_score"] = {"J": sc["J"].clone(), "iters": r["iters_done"].clone()}
+        for j, (h, nu) in enumerate(rand):
+            out[f"random{j}"] = {"J": dtp.chain_score(S_up, Sd, h, nu, D, workspace=ws, check=check)["J"].clone()}
+        return out
+
+    run(True)
+    torch.cuda.synchronize()
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    res = run(False)
+    s1.record(stream)
+    torch.cuda.synchronize()
+    if dtp.workspace_status(ws) != dtp.DTP_OK:
+        raise RuntimeError("layout suite reported a device-side error")
+    J = {k: round(float(v["J"]), 4) for k, v in res.items()}
+    rnd = [J[f"random{j}"] for j in range(8)]
+    return {"D": D, "ms": s0.elapsed_time(s1), "J": {k: v for k, v in J.items() if not k.startswith("random")},
+            "J_random_mean": round(sum(rnd) / len(rnd), 4), "J_random_range": [min(rnd), max(rnd)],
+            "J_random_expected": (2 * Lyr - 1) / D,
+            "layouts": len(res)}
+
+
 def run_model(args):
     """Whole-model pipeline timing: every layer's affinity pass with the down-edge term on all
     its tokens, the ||w^d||^2 finalize, ||b_gk||^2 and S_down, then the whole-model search per D.
@@ -200,10 +251,15 @@ def run_model(args):
     Lyr, G, N, T, d = w.layers, w.G, w.N, w.T, w.d
     S_up = torch.empty((Lyr, G, N), dtype=torch.float32, device=dev)
     S_down = torch.empty((max(Lyr - 1, 1), G, N), dtype=torch.float32, device=dev)
-    ws = dtp.affinity_workspace(T, d, G, N, dtp.DTP_BF16, dev)
-    t_aff = t_down = 0.0
+    ws = dtp.affinity_workspace(T, d, G, N, dtp.DTP_BF16, dev) if args.qheads == 1 else \
+        torch.empty(dtp.affinity_grouped_workspace_size(T, d, G * args.qheads, args.qheads, N, dtp.DTP_BF16),
+                    dtype=torch.uint8, device=dev)
+    S_add = torch.zeros((Lyr, G, N), dtype=torch.float32, device=dev) if args.add_score else None
+    t_aff = t_down = t_add = 0.0
+    q = args.qheads
     for i in range(Lyr):
-        L = synth.make_workload_layer(w, i, device=dev)
+        L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
+            synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
         Dn = synth.make_down_inputs(d, G, w.qkv_rows, N, T, seed=w.seed + 1000 + i, device=dev)
         act2 = torch.zeros(N, dtype=torch.float32, device=dev)
         A = S_up[i]
@@ -211,16 +267,30 @@ def run_model(args):
         torch.cuda.synchronize()
         e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
         e0.record(stream)
-        dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"], A=A, act2=act2, workspace=ws)
+        if q == 1:
+            dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"], A=A, act2=act2,
+                                         workspace=ws)
+        else:   # one row of C per query head, summed over each KV group's q query heads
+            dtp.affinity_accumulate_grouped(L["X"], L["C"], L["W_gate"], L["W_up"], q, A=A, rms_next=Dn["rms"],
+                                            act2=act2, workspace=ws)
         dtp.affinity_finalize(A, T, dtp.down_sqnorm(Dn["W_down"]))
         e1.record(stream)
         if i + 1 < Lyr:
             bn = dtp.down_weight_sqnorm(Dn["Wqkv"], Dn["gamma"], Dn["W_down"])
             S_down[i].copy_(dtp.down_finalize(act2, bn, T))
         e2.record(stream)
+        if args.add_score:
+            e3 = torch.cuda.Event(enable_timing=True)
+            if q == 1:
+                dtp.affinity_add_accumulate(L["C"], L["W_gate"], L["W_up"], A_add=S_add[i])
+            else:
+                dtp.affinity_add_accumulate_grouped(L["C"], L["W_gate"], L["W_up"], q, A_add=S_add[i])
+            e3.record(stream)
         torch.cuda.synchronize()
         t_aff += e0.elapsed_time(e1)
         t_down += e1.elapsed_time(e2)
+        if args.add_score:
+            t_add += e2.elapsed_time(e3)
         del L, Dn
     if dtp.workspace_status(ws) != dtp.DTP_OK:
         raise RuntimeError("affinity kernel reported a device-side error")
@@ -236,14 +306,18 @@ def run_model(args):
         torch.cuda.synchronize()
         searches[f"D{D}"] = {"ms": s0.elapsed_time(s1) / 3, "J": float(r["J"]), "J_random": (2 * Lyr - 1) / D,
                              "iters_done": int(r["iters_done"])}
+    suite = layout_suite(args, w, S_up, S_down, S_add if args.add_score else None, stream)
     total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values())
-    fl = 2.0 * d * 2 * N * (G + 1) * T * Lyr
+    chunk = (16 // q) * q                      # query heads per launch; each launch has its own X pass
+    fl = 2.0 * d * 2 * N * (G * q + -(-(G * q) // chunk)) * T * Lyr
     line = {"metric": f"whole-model affinity + layout time ({args.model})", "value": total_ms / 1e3, "unit": "s",
             "higher_is_better": False, "n_gpus": 1, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": args.model, "layers": Lyr, "d": d, "G": G, "N": N, "T_per_layer": T,
+                       "query_heads_per_group": q,
                        "D": list(w.D), "iters": w.iters, "qkv_rows": w.qkv_rows},
             "affinity_ms": t_aff, "affinity_tflops": fl / (t_aff / 1e3) / 1e12,
             "layer_tokens_per_s": Lyr * T / (t_aff / 1e3), "down_edge_ms": t_down, "search": searches,
+            "add_affinity_ms": t_add if args.add_score else None, "layout_suite": suite,
             "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s"}
     print(json.dumps(line), flush=True)
 
@@ -258,6 +332,9 @@ def main():
     ap.add_argument("--cpu-tokens", type=int, default=64, help="token slice per step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--model", default=None, help="time a whole-model pipeline instead, e.g. qwen3_0.6b_model")
+    ap.add_argument("--add-score", action="store_true", help="with --model: also the ADD affinity and its layout")
+    ap.add_argument("--qheads", type=int, default=1,
+                    help="with --model: query heads per KV group; >1 scores each query head and sums per group")
     args = ap.parse_args()
     w = synth.WORKLOADS[WORKLOAD]
     if args.model:

@@ -111,6 +111,35 @@ int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate,
                                void* stream);
 
 /*
+ * The first-order score per query head, summed over the query heads of each
+ * KV group (Sec. 3, "Affinity scores": E_t[Delta_hk^2] is taken per query head
+ * h from that head's own write p_h, and the group's score is the sum of its
+ * query heads' scores):
+ *   A[g,k] += sum over h = g*q_per_group .. (g+1)*q_per_group - 1 of
+ *             sum_t Delta_{t,h,k}^2
+ * This is a sum of squares, not the square of the group's summed write that
+ * dtp_affinity_accumulate takes when given one C row per KV group.
+ *   X, W_gate, W_up, rms_next, act2, dtype: as dtp_affinity_accumulate_ex
+ *   C_q          [H_q, T, d], device: each query head's write p_h into the
+ *                residual (the head's slice of W_o applied to its output)
+ *   H_q          query heads, 1..128, a multiple of q_per_group
+ *   q_per_group  query heads per KV group (1..16); H_q / q_per_group <= 16
+ *   A            [H_q / q_per_group, N] fp32, device, accumulated into
+ * Query heads are processed in chunks of at most 16 (whole groups); the X
+ * pass runs once per chunk and act2 (when requested) is added once.  Row g's
+ * sum runs over its query heads in order, then token tiles, so the result is
+ * deterministic; with q_per_group == 1 it equals dtp_affinity_accumulate_ex.
+ * Workspace from dtp_affinity_grouped_workspace_size.  Errors as
+ * dtp_affinity_accumulate_ex.
+ */
+int dtp_affinity_grouped_workspace_size(int64_t T, int d, int H_q, int q_per_group, int N, int dtype,
+                                        size_t* bytes);
+int dtp_affinity_accumulate_grouped(const void* X, const void* C_q, const void* W_gate, const void* W_up,
+                                    const float* rms_next, int64_t T, int d, int H_q, int q_per_group, int N,
+                                    int dtype, float* A, float* act2, void* workspace, size_t workspace_bytes,
+                                    void* stream);
+
+/*
  * The ADD score of Sec. 3 before the mean: the squared additive contribution
  * of KV group h's piece to neuron k's pre-activations, ignoring the operating
  * point and ||w^d_k||:
@@ -123,6 +152,20 @@ int dtp_affinity_add_workspace_size(int64_t T, int d, int H_kv, int N, size_t* b
 int dtp_affinity_add_accumulate(const void* C, const void* W_gate, const void* W_up, int64_t T, int d,
                                 int H_kv, int N, float* A_add, void* workspace,
                                 size_t workspace_bytes, void* stream);
+
+/*
+ * The ADD score per query head, summed over the query heads of each KV group
+ * (Sec. 3):  A_add[g,k] += sum over the group's query heads h of
+ *            sum_t (p_{h,t} . w^g_k)^2 + (p_{h,t} . w^u_k)^2
+ * C_q [H_q, T, d] bf16 (each query head's write), A_add [H_q / q_per_group, N]
+ * fp32 accumulated; H_q and q_per_group as dtp_affinity_accumulate_grouped.
+ * Workspace from dtp_affinity_add_grouped_workspace_size.  Deterministic;
+ * with q_per_group == 1 equals dtp_affinity_add_accumulate.  Asynchronous.
+ */
+int dtp_affinity_add_grouped_workspace_size(int64_t T, int d, int H_q, int q_per_group, int N, size_t* bytes);
+int dtp_affinity_add_accumulate_grouped(const void* C_q, const void* W_gate, const void* W_up, int64_t T, int d,
+                                        int H_q, int q_per_group, int N, float* A_add, void* workspace,
+                                        size_t workspace_bytes, void* stream);
 
 /*
  * Down-edge weight factor (Sec. 3): bn[g,k] = ||b_gk||^2 with
@@ -292,6 +335,47 @@ int dtp_search_chain_workspace_size(int layers, int H_kv, int N, int D, size_t* 
 int dtp_search_chain(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D,
                      int iters, int32_t* head_part, int32_t* neuron_dev, int64_t* J_q, double* J,
                      int32_t* iters_done, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * dtp_search_chain with the ablations of Sec. 3 ("Optimiser"; the layouts of
+ * Table 4): restricting which layers move, freezing heads or neurons, or
+ * minimising J (the anti-optimised layout).
+ *   move_heads    [layers] uint8, device, or NULL (= every layer): 0 keeps
+ *                 layer i's head partition at the contiguous start
+ *   move_neurons  [layers] uint8, device, or NULL: 0 keeps layer i's neuron
+ *                 assignment contiguous (nu_i(k) = floor(k D / N))
+ *   minimize      nonzero: every step minimises J exactly given the other
+ *                 block (ties: lexicographically smallest, as when
+ *                 maximising); the stop rule applies to -J
+ * dtp_search_chain(...) equals dtp_search_chain_ex(..., NULL, NULL, 0, ...).
+ * The flag arrays are read by the kernels, so they must stay valid until the
+ * stream reaches the end of this call's work.  Same workspace and errors as
+ * dtp_search_chain.
+ */
+int dtp_search_chain_ex(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D, int iters,
+                        const uint8_t* move_heads, const uint8_t* move_neurons, int minimize, int32_t* head_part,
+                        int32_t* neuron_dev, int64_t* J_q, double* J, int32_t* iters_done, void* workspace,
+                        size_t workspace_bytes, void* stream);
+
+/*
+ * J of a given layout (Eq. objective, both sums) and its per-edge terms; the
+ * paper scores random layouts this way alongside the optimiser (Sec. 3).
+ *   head_part   [layers, H_kv] int32, device, entries in [0, D)
+ *   neuron_dev  [layers, N] int32, device, entries in [0, D)
+ *   edge_q      [2*layers - 1] int64 out, device, or NULL: edge 2i is the
+ *               co-located mass of layer i's up edge, edge 2i+1 that of its
+ *               down edge, each in units of 2^-43 of that edge's own total
+ *               (edge_q / 2^43 is the co-located fraction of the edge)
+ *   J_q, J      the sum, as in dtp_search_chain
+ * The layout need not be balanced.  S_up, S_down and the size rules are those
+ * of dtp_search_chain (D as given); workspace from
+ * dtp_search_chain_workspace_size.  Asynchronous; negative or non-finite
+ * affinities and layout entries outside [0, D) are reported as DTP_ERR_ARG
+ * through the workspace status word.
+ */
+int dtp_chain_score(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D,
+                    const int32_t* head_part, const int32_t* neuron_dev, int64_t* edge_q, int64_t* J_q, double* J,
+                    void* workspace, size_t workspace_bytes, void* stream);
 
 #ifdef __cplusplus
 }

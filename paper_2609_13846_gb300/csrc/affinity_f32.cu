@@ -137,15 +137,20 @@ affinity_fo_f32_kernel(const float* __restrict__ X, const float* __restrict__ C,
     }
 }
 
+// A[g,k] += sum over heads h of row g (qpg consecutive heads) and token tiles, head by head.
 __global__ void f32_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
-                                  int64_t tiles, const float* __restrict__ partial_act, float* __restrict__ act2) {
-    const int64_t total_a = static_cast<int64_t>(G) * N;
+                                  int64_t tiles, const float* __restrict__ partial_act, float* __restrict__ act2,
+                                  int qpg) {
+    const int64_t heads_n = static_cast<int64_t>(G) * N;
+    const int64_t total_a = static_cast<int64_t>(G / qpg) * N;
     const int64_t total = total_a + (act2 ? N : 0);
     for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
          idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         float s = 0.0f;
         if (idx < total_a) {
-            for (int64_t t = 0; t < tiles; ++t) s += partial[t * total_a + idx];
+            const int64_t g = idx / N, k = idx % N;
+            for (int64_t h = g * qpg; h < (g + 1) * qpg; ++h)
+                for (int64_t t = 0; t < tiles; ++t) s += partial[t * heads_n + h * N + k];
             A[idx] += s;
         } else {
             const int64_t k = idx - total_a;
@@ -161,8 +166,9 @@ size_t workspace_bytes(int64_t T, int d, int G, int N) {
     return kWorkspaceHeader + static_cast<size_t>(tiles) * (G + 1) * N * sizeof(float);
 }
 
-int launch(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
-           float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2) {
+int launch_grouped(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
+                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg) {
+    if (qpg < 1 || G % qpg) return DTP_ERR_ARG;
     const int64_t tiles = (T + TT - 1) / TT;
     if (tiles > 65535) return DTP_ERR_UNSUPPORTED;
     float* partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(workspace) + kWorkspaceHeader);
@@ -172,11 +178,17 @@ int launch(const float* X, const float* C, const float* Wg, const float* Wu, int
     affinity_fo_f32_kernel<<<grid, kThreads, 0, stream>>>(X, C, Wg, Wu, T, d, G, N, partial,
                                                           want_act ? rms : nullptr, partial_act);
     DTP_CUDA_TRY(cudaGetLastError());
-    const int64_t total = static_cast<int64_t>(G) * N + (want_act ? N : 0);
+    const int64_t total = static_cast<int64_t>(G / qpg) * N + (want_act ? N : 0);
     const int blocks = static_cast<int>((total + 255) / 256 < 1024 ? (total + 255) / 256 : 1024);
-    f32_reduce_kernel<<<blocks, 256, 0, stream>>>(partial, A, G, N, tiles, partial_act, want_act ? act2 : nullptr);
+    f32_reduce_kernel<<<blocks, 256, 0, stream>>>(partial, A, G, N, tiles, partial_act, want_act ? act2 : nullptr,
+                                                  qpg);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
+}
+
+int launch(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
+           float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2) {
+    return launch_grouped(X, C, Wg, Wu, T, d, G, N, A, workspace, stream, rms, act2, 1);
 }
 
 // S_down[g,k] = act2[k] / T_total * bn[g,k]

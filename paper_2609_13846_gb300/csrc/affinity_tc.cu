@@ -402,14 +402,17 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
     if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, static_cast<int>(DTP_ERR_NOT_CONVERGED));
 }
 
-// A[h,k] += sum over token chunks of the unit partials.  Eight threads share
-// one output: thread s sums the chunks c = s, s+8, ..., then the eight sums
-// are added in a fixed order, so the result does not depend on scheduling.
+// A[g,k] += sum over the heads h of row g (h = g*qpg ... g*qpg + qpg - 1) and
+// over token chunks of the unit partials; qpg = 1 gives one row per head, qpg
+// > 1 sums the query heads of a KV group (Sec. 3, per-query-head scores).
+// Eight threads share one output: thread s sums the chunks c = s, s+8, ...
+// (head by head), then the eight sums are added in a fixed order, so the
+// result does not depend on scheduling.
 constexpr int kReduceSplit = 8;
 __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
                                        int NT, int TC, const float* __restrict__ partial_act,
-                                       float* __restrict__ act2) {
-    const int64_t total_a = static_cast<int64_t>(G) * N;
+                                       float* __restrict__ act2, int qpg) {
+    const int64_t total_a = static_cast<int64_t>(G / qpg) * N;
     const int64_t total = total_a + (act2 ? N : 0);
     const int s = threadIdx.x % kReduceSplit;
     const int64_t per_block = blockDim.x / kReduceSplit;
@@ -417,11 +420,12 @@ __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float*
         const int64_t idx = base + threadIdx.x / kReduceSplit;
         float sum = 0.0f;
         if (idx < total_a) {
-            const int h = static_cast<int>(idx / N);
+            const int g = static_cast<int>(idx / N);
             const int k = static_cast<int>(idx % N);
             const int j = k / BNEU, r = k % BNEU;
-            for (int c = s; c < TC; c += kReduceSplit)
-                sum += partial[((static_cast<int64_t>(c) * NT + j) * G + h) * BNEU + r];
+            for (int h = g * qpg; h < (g + 1) * qpg; ++h)
+                for (int c = s; c < TC; c += kReduceSplit)
+                    sum += partial[((static_cast<int64_t>(c) * NT + j) * G + h) * BNEU + r];
         } else if (idx < total) {
             const int k = static_cast<int>(idx - total_a);
             const int j = k / BNEU, r = k % BNEU;
@@ -484,8 +488,10 @@ size_t workspace_bytes_with_act(int64_t T, int d, int G, int N) {
     return align_up(workspace_bytes(T, d, G, N), 256) + static_cast<size_t>(NT * TC) * BNEU * sizeof(float);
 }
 
-int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
-           void* workspace, cudaStream_t stream, const float* rms, float* act2) {
+// G heads of C; A receives G / qpg rows (qpg consecutive heads summed per row).
+int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N,
+                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg) {
+    if (qpg < 1 || G % qpg) return DTP_ERR_ARG;
     CUtensorMap m_wg, m_wu, m_x, m_c;
     const cuuint64_t row_stride = static_cast<cuuint64_t>(d) * 2;
     cuuint64_t dw[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(N)};
@@ -532,14 +538,19 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
     p.tail_items = left * p.split;
     affinity_fo_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(m_wg, m_wu, m_x, m_c, p);
     DTP_CUDA_TRY(cudaGetLastError());
-    const int64_t total = static_cast<int64_t>(G) * N + (p.rms ? N : 0);
+    const int64_t total = static_cast<int64_t>(G / qpg) * N + (p.rms ? N : 0);
     const int64_t outs_per_block = 256 / kReduceSplit;
     const int64_t want = (total + outs_per_block - 1) / outs_per_block;
     const int rblocks = static_cast<int>(want < 8 * sms ? want : 8 * sms);
     affinity_reduce_kernel<<<rblocks, 256, 0, stream>>>(p.partial, A, G, N, p.NT, p.TC, p.partial_act,
-                                                        p.rms ? act2 : nullptr);
+                                                        p.rms ? act2 : nullptr, qpg);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
+}
+
+int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
+           void* workspace, cudaStream_t stream, const float* rms, float* act2) {
+    return launch_grouped(X, C, Wg, Wu, T, d, G, N, A, workspace, stream, rms, act2, 1);
 }
 
 }  // namespace tc

@@ -11,11 +11,15 @@ size_t workspace_bytes(int64_t T, int d, int G, int N);
 size_t workspace_bytes_with_act(int64_t T, int d, int G, int N);
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
            void* workspace, cudaStream_t stream, const float* rms, float* act2);
+int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N,
+                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg);
 }  // namespace tc
 namespace f32 {
 size_t workspace_bytes(int64_t T, int d, int G, int N);
 int launch(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
            float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2);
+int launch_grouped(const float* X, const float* C, const float* Wg, const float* Wu, int64_t T, int d, int G, int N,
+                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg);
 }  // namespace f32
 namespace sq {
 size_t down_workspace_bytes(int G, int R, int d, int N);
@@ -24,6 +28,8 @@ int launch_down(const void* Wqkv, const void* gamma, const void* Wd, int G, int 
 size_t add_workspace_bytes(int64_t T, int G, int N);
 int launch_add(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
                void* workspace, cudaStream_t stream);
+int launch_add_grouped(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
+                       void* workspace, cudaStream_t stream, int qpg);
 }  // namespace sq
 int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream);
 int launch_down_finalize(const float* act2, const float* bn, int G, int N, int64_t T_total, float* S,
@@ -35,8 +41,12 @@ int64_t partition_count(int G, int D);
 int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* head, int32_t* nu, int64_t* score_q,
            double* score, int32_t* iters_done, void* workspace, cudaStream_t stream);
 size_t chain_workspace_bytes(int Lyr, int G, int N, int D);
-int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters, int32_t* head,
-                 int32_t* nu, int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream);
+int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters,
+                 const uint8_t* move_heads, const uint8_t* move_neurons, int minimize, int32_t* head, int32_t* nu,
+                 int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream);
+int launch_chain_score(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, const int32_t* head,
+                       const int32_t* nu, int64_t* edge_q, int64_t* J_q, double* J, void* workspace,
+                       cudaStream_t stream);
 }  // namespace search
 }  // namespace dtp
 
@@ -57,6 +67,19 @@ bool affinity_sizes_ok(int64_t T, int d, int H, int N, int dtype) {
 size_t affinity_ws(int64_t T, int d, int H, int N, int dtype, bool with_act) {
     if (dtype != DTP_BF16) return f32::workspace_bytes(T, d, H, N);
     return with_act ? tc::workspace_bytes_with_act(T, d, H, N) : tc::workspace_bytes(T, d, H, N);
+}
+
+// Query heads per launch of the grouped affinity: the largest multiple of qpg within kMaxHeads.
+constexpr int kMaxQueryHeads = 128;
+int grouped_chunk(int H_q, int qpg) {
+    const int c = (kMaxHeads / qpg) * qpg;
+    return H_q < c ? H_q : c;
+}
+
+bool grouped_sizes_ok(int64_t T, int d, int H_q, int qpg, int N, int dtype) {
+    if (qpg < 1 || qpg > kMaxHeads || H_q < 1 || H_q > kMaxQueryHeads || H_q % qpg || H_q / qpg > kMaxHeads)
+        return false;
+    return affinity_sizes_ok(T, d, grouped_chunk(H_q, qpg), N, dtype);
 }
 
 bool search_sizes_ok(int layers, int H, int N, int D, int iters) {
@@ -118,6 +141,48 @@ int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, co
                                       workspace_bytes, stream);
 }
 
+int dtp_affinity_grouped_workspace_size(int64_t T, int d, int H_q, int q_per_group, int N, int dtype,
+                                        size_t* bytes) {
+    if (!bytes || !grouped_sizes_ok(T, d, H_q, q_per_group, N, dtype)) return DTP_ERR_ARG;
+    *bytes = affinity_ws(T, d, grouped_chunk(H_q, q_per_group), N, dtype, true);
+    return DTP_OK;
+}
+
+int dtp_affinity_accumulate_grouped(const void* X, const void* C_q, const void* W_gate, const void* W_up,
+                                    const float* rms_next, int64_t T, int d, int H_q, int q_per_group, int N,
+                                    int dtype, float* A, float* act2, void* workspace, size_t workspace_bytes,
+                                    void* stream) {
+    if (!grouped_sizes_ok(T, d, H_q, q_per_group, N, dtype)) return DTP_ERR_ARG;
+    if ((rms_next == nullptr) != (act2 == nullptr)) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;
+    if (!X || !C_q || !W_gate || !W_up || !A) return DTP_ERR_ARG;
+    if (!aligned16(X) || !aligned16(C_q) || !aligned16(W_gate) || !aligned16(W_up) || !aligned16(A))
+        return DTP_ERR_ARG;
+    const bool with_act = act2 != nullptr;
+    if (with_act && (!aligned16(act2) || !aligned16(rms_next))) return DTP_ERR_ARG;
+    const int chunk = grouped_chunk(H_q, q_per_group);
+    const size_t need = affinity_ws(T, d, chunk, N, dtype, with_act);
+    if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    const size_t elem = dtype == DTP_BF16 ? 2 : 4;
+    // chunks of whole KV groups; each chunk's C block starts 16-byte aligned (d % 8 == 0)
+    for (int h0 = 0; h0 < H_q; h0 += chunk) {
+        const int hc = H_q - h0 < chunk ? H_q - h0 : chunk;
+        const void* Cc = static_cast<const uint8_t*>(C_q) + static_cast<size_t>(h0) * T * d * elem;
+        float* Ac = A + static_cast<int64_t>(h0 / q_per_group) * N;
+        const float* r = h0 == 0 ? rms_next : nullptr;   // the activation term once, with the first chunk
+        float* a2 = h0 == 0 ? act2 : nullptr;
+        const int st = dtype == DTP_BF16
+                           ? tc::launch_grouped(X, Cc, W_gate, W_up, T, d, hc, N, Ac, workspace, s, r, a2, q_per_group)
+                           : f32::launch_grouped(static_cast<const float*>(X), static_cast<const float*>(Cc),
+                                                 static_cast<const float*>(W_gate), static_cast<const float*>(W_up), T,
+                                                 d, hc, N, Ac, workspace, s, r, a2, q_per_group);
+        if (st != DTP_OK) return st;
+    }
+    return DTP_OK;
+}
+
 int dtp_affinity_add_workspace_size(int64_t T, int d, int H_kv, int N, size_t* bytes) {
     if (!bytes || !affinity_sizes_ok(T, d, H_kv, N, DTP_BF16)) return DTP_ERR_ARG;
     *bytes = sq::add_workspace_bytes(T, H_kv, N);
@@ -136,6 +201,35 @@ int dtp_affinity_add_accumulate(const void* C, const void* W_gate, const void* W
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
     return sq::launch_add(C, W_gate, W_up, T, d, H_kv, N, A_add, workspace, s);
+}
+
+int dtp_affinity_add_grouped_workspace_size(int64_t T, int d, int H_q, int q_per_group, int N, size_t* bytes) {
+    if (!bytes || !grouped_sizes_ok(T, d, H_q, q_per_group, N, DTP_BF16)) return DTP_ERR_ARG;
+    *bytes = sq::add_workspace_bytes(T, grouped_chunk(H_q, q_per_group), N);
+    return DTP_OK;
+}
+
+int dtp_affinity_add_accumulate_grouped(const void* C_q, const void* W_gate, const void* W_up, int64_t T, int d,
+                                        int H_q, int q_per_group, int N, float* A_add, void* workspace,
+                                        size_t workspace_bytes, void* stream) {
+    if (!grouped_sizes_ok(T, d, H_q, q_per_group, N, DTP_BF16)) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;
+    if (!C_q || !W_gate || !W_up || !A_add || !aligned16(C_q) || !aligned16(W_gate) || !aligned16(W_up) ||
+        !aligned16(A_add))
+        return DTP_ERR_ARG;
+    const int chunk = grouped_chunk(H_q, q_per_group);
+    if (!workspace || workspace_bytes < sq::add_workspace_bytes(T, chunk, N) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    for (int h0 = 0; h0 < H_q; h0 += chunk) {
+        const int hc = H_q - h0 < chunk ? H_q - h0 : chunk;
+        const void* Cc = static_cast<const uint8_t*>(C_q) + static_cast<size_t>(h0) * T * d * 2;
+        const int st = sq::launch_add_grouped(Cc, W_gate, W_up, T, d, hc, N, A_add + static_cast<int64_t>(h0 / q_per_group) * N,
+                                              workspace, s, q_per_group);
+        if (st != DTP_OK) return st;
+    }
+    return DTP_OK;
 }
 
 int dtp_down_weight_workspace_size(int H_kv, int R, int d, int N, size_t* bytes) {
@@ -206,17 +300,38 @@ int dtp_search_chain_workspace_size(int layers, int H_kv, int N, int D, size_t* 
     return DTP_OK;
 }
 
-int dtp_search_chain(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D, int iters,
-                     int32_t* head_part, int32_t* neuron_dev, int64_t* J_q, double* J, int32_t* iters_done,
-                     void* workspace, size_t workspace_bytes, void* stream) {
+int dtp_search_chain_ex(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D, int iters,
+                        const uint8_t* move_heads, const uint8_t* move_neurons, int minimize, int32_t* head_part,
+                        int32_t* neuron_dev, int64_t* J_q, double* J, int32_t* iters_done, void* workspace,
+                        size_t workspace_bytes, void* stream) {
     if (!search_sizes_ok(layers, H_kv, N, D, iters)) return DTP_ERR_ARG;
     if (!S_up || (layers > 1 && !S_down) || !head_part || !neuron_dev || !J_q || !J || !iters_done)
         return DTP_ERR_ARG;
     if (!aligned16(S_up) || (S_down && !aligned16(S_down))) return DTP_ERR_ARG;
     if (!workspace || workspace_bytes < search::chain_workspace_bytes(layers, H_kv, N, D) || !aligned16(workspace))
         return DTP_ERR_WORKSPACE;
-    return search::launch_chain(S_up, S_down, layers, H_kv, N, D, iters, head_part, neuron_dev, J_q, J, iters_done,
-                                workspace, static_cast<cudaStream_t>(stream));
+    return search::launch_chain(S_up, S_down, layers, H_kv, N, D, iters, move_heads, move_neurons, minimize,
+                                head_part, neuron_dev, J_q, J, iters_done, workspace,
+                                static_cast<cudaStream_t>(stream));
+}
+
+int dtp_search_chain(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D, int iters,
+                     int32_t* head_part, int32_t* neuron_dev, int64_t* J_q, double* J, int32_t* iters_done,
+                     void* workspace, size_t workspace_bytes, void* stream) {
+    return dtp_search_chain_ex(S_up, S_down, layers, H_kv, N, D, iters, nullptr, nullptr, 0, head_part, neuron_dev,
+                               J_q, J, iters_done, workspace, workspace_bytes, stream);
+}
+
+int dtp_chain_score(const float* S_up, const float* S_down, int layers, int H_kv, int N, int D,
+                    const int32_t* head_part, const int32_t* neuron_dev, int64_t* edge_q, int64_t* J_q, double* J,
+                    void* workspace, size_t workspace_bytes, void* stream) {
+    if (!search_sizes_ok(layers, H_kv, N, D, 1)) return DTP_ERR_ARG;
+    if (!S_up || (layers > 1 && !S_down) || !head_part || !neuron_dev || !J_q || !J) return DTP_ERR_ARG;
+    if (!aligned16(S_up) || (S_down && !aligned16(S_down))) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < search::chain_workspace_bytes(layers, H_kv, N, D) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
+    return search::launch_chain_score(S_up, S_down, layers, H_kv, N, D, head_part, neuron_dev, edge_q, J_q, J,
+                                      workspace, static_cast<cudaStream_t>(stream));
 }
 
 int dtp_search_layout(const float* A, int H_kv, int N, int D, int iters, int32_t* head_part, int32_t* neuron_dev,

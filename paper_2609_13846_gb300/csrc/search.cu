@@ -687,8 +687,16 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
 // step given all neuron assignments (column sums over nu_i for the up edge and
 // nu_{i-1} for the down edge), then the score.  Each step maximises J exactly
 // given the other block, so layers run in parallel, one block each.  A device
-// flag stops later iterations after the first one without a strict increase,
-// so the host never waits.
+// flag stops later iterations after the first one (after the first) without a
+// strict increase, so the host never waits.
+//
+// Ablations (Sec. 3 "Optimiser", Table 4): per-layer flags freeze a layer's
+// heads or neurons at the contiguous start, and `minimize` minimises J.  A
+// minimising step maximises R - gain with R the per-neuron (per-head) sum of
+// the gains over devices: every neuron (head) sits on exactly one device, so
+// the offset shifts all assignments' totals equally and leaves the set of
+// optimal assignments (hence the canonical one) unchanged, while keeping every
+// gain non-negative and below 2^44 as the exact steps require.
 
 constexpr int kNormBits = 43;   // gains (one up + one down matrix) stay below 2^44
 constexpr int kNormPreBits = 40;
@@ -702,22 +710,27 @@ struct ChainState {
 __global__ void chain_init_kernel(ChainState* st, int64_t* J_q, double* J, int32_t* iters_done) {
     st->done = 0;
     st->iters = 0;
-    st->prev = -1;
+    st->prev = INT64_MIN;
     *J_q = 0;
     *J = 0.0;
-    *iters_done = 0;
+    if (iters_done) *iters_done = 0;
 }
 
 // One block per matrix: m < L is the up edge of layer m, m >= L the down edge of layer m - L.
+// head / nu (may be null) receive the contiguous start layout.
 __global__ void __launch_bounds__(kThreads, 1)
 chain_normalize_kernel(const float* __restrict__ S_up, const float* __restrict__ S_down, int L, int G, int N, int D,
-                       int64_t* __restrict__ nbuf, int32_t* __restrict__ head, ChainState* st, int* ws_status) {
+                       int64_t* __restrict__ nbuf, int32_t* __restrict__ head, int32_t* __restrict__ nu,
+                       ChainState* st, int* ws_status) {
     __shared__ Shared sh;
     const int m = blockIdx.x;
     const int64_t GN = static_cast<int64_t>(G) * N;
     const float* src = m < L ? S_up + m * GN : S_down + (m - L) * GN;
     int64_t* dst = nbuf + m * GN;
-    if (m < L && threadIdx.x < G) head[m * G + threadIdx.x] = (threadIdx.x * D) / G;
+    if (m < L && head && threadIdx.x < G) head[m * G + threadIdx.x] = (threadIdx.x * D) / G;
+    if (m < L && nu)
+        for (int k = threadIdx.x; k < N; k += kThreads)
+            nu[static_cast<int64_t>(m) * N + k] = static_cast<int>((static_cast<int64_t>(k) * D) / N);
     uint32_t amax_bits = 0;
     int bad = 0;
     for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
@@ -746,10 +759,11 @@ chain_normalize_kernel(const float* __restrict__ S_up, const float* __restrict__
     }
 }
 
-// M[k,l] = up mass of k from heads of layer i on l + down mass of k into heads of layer i+1 on l.
+// M[k,l] = up mass of k from heads of layer i on l + down mass of k into heads of layer i+1 on l;
+// minimising: sum_l' M[k,l'] - M[k,l].
 template <int DT>
 __device__ void build_gain_chain(const Layer& L, Shared& sh, const int64_t* __restrict__ nU,
-                                 const int64_t* __restrict__ nD) {
+                                 const int64_t* __restrict__ nD, bool minimize) {
     for (int k = threadIdx.x; k < L.N; k += kThreads) {
         int64_t m[DT];
 #pragma unroll
@@ -761,8 +775,13 @@ __device__ void build_gain_chain(const Layer& L, Shared& sh, const int64_t* __re
 #pragma unroll
             for (int l = 0; l < DT; ++l) m[l] += (l == hg ? u : 0) + (l == hn ? dn : 0);
         }
+        int64_t r = 0;
+        if (minimize) {
 #pragma unroll
-        for (int l = 0; l < DT; ++l) L.M[static_cast<int64_t>(k) * DT + l] = m[l];
+            for (int l = 0; l < DT; ++l) r += m[l];
+        }
+#pragma unroll
+        for (int l = 0; l < DT; ++l) L.M[static_cast<int64_t>(k) * DT + l] = minimize ? r - m[l] : m[l];
     }
     __syncthreads();
 }
@@ -806,11 +825,13 @@ template <int DT>
 __global__ void __launch_bounds__(kThreads, 1)
 chain_neuron_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, const int32_t* __restrict__ head,
                     int32_t* __restrict__ nu_out, int64_t* __restrict__ prices, ChainState* st, int* ws_status,
-                    uint8_t* __restrict__ gbuf, size_t per_layer, int use_smem) {
+                    uint8_t* __restrict__ gbuf, size_t per_layer, int use_smem,
+                    const uint8_t* __restrict__ move_neurons, int minimize) {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ Shared sh;
     if (*reinterpret_cast<volatile int*>(&st->done)) return;
     const int i = blockIdx.x;
+    if (move_neurons && !move_neurons[i]) return;   // frozen: nu_i stays contiguous
     const int64_t GN = static_cast<int64_t>(G) * N;
     uint8_t* buf = use_smem ? dsm : gbuf + static_cast<size_t>(i) * per_layer;
     Layer L;
@@ -830,7 +851,7 @@ chain_neuron_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, con
     if (threadIdx.x < DMAX) sh.pi[threadIdx.x] = prices[i * DMAX + threadIdx.x];
     if (threadIdx.x == 0) sh.status = DTP_OK;
     __syncthreads();
-    build_gain_chain<DT>(L, sh, nbuf + i * GN, has_down ? nbuf + (Lyr + i) * GN : nullptr);
+    build_gain_chain<DT>(L, sh, nbuf + i * GN, has_down ? nbuf + (Lyr + i) * GN : nullptr, minimize != 0);
     if constexpr (DT == 2) neuron_step_d2(L, sh);
     else neuron_step_general<DT>(L, sh);
     __syncthreads();
@@ -848,7 +869,8 @@ chain_neuron_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, con
 template <int DT>
 __global__ void __launch_bounds__(kThreads, 1)
 chain_head_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, const int32_t* __restrict__ nu_all,
-                  int32_t* __restrict__ head, int64_t* __restrict__ layer_score, ChainState* st, uint32_t n_parts) {
+                  int32_t* __restrict__ head, int64_t* __restrict__ layer_score, ChainState* st, uint32_t n_parts,
+                  const uint8_t* __restrict__ move_heads, int minimize) {
     __shared__ Shared sh;
     if (*reinterpret_cast<volatile int*>(&st->done)) return;
     const int i = blockIdx.x;
@@ -865,22 +887,93 @@ chain_head_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, const
     head_sums_chain<DT>(L, sh, nbuf + i * GN, nu_all + static_cast<int64_t>(i) * N,
                         i > 0 ? nbuf + (Lyr + i - 1) * GN : nullptr,
                         i > 0 ? nu_all + static_cast<int64_t>(i - 1) * N : nullptr);
+    const int64_t sign = minimize ? -1 : 1;
+    if (move_heads && !move_heads[i]) {            // frozen: score the current (contiguous) partition
+        if (threadIdx.x == 0) {
+            int64_t sc = 0;
+            for (int g = 0; g < G; ++g) sc += sh.B[g * DT + head[i * G + g]];
+            layer_score[i] = sign * sc;
+        }
+        return;
+    }
+    int64_t R = 0;                                  // sum_g R_g, held by thread 0
+    if (minimize) {
+        if (threadIdx.x < G) {
+            int64_t r = 0;
+#pragma unroll
+            for (int l = 0; l < DT; ++l) r += sh.B[threadIdx.x * DT + l];
+#pragma unroll
+            for (int l = 0; l < DT; ++l) sh.B[threadIdx.x * DT + l] = r - sh.B[threadIdx.x * DT + l];
+            sh.red_i64[threadIdx.x] = r;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0)
+            for (int g = 0; g < G; ++g) R += sh.red_i64[g];
+        __syncthreads();                            // choose_partition reuses red_i64
+    }
     choose_partition(L, sh, n_parts);
     if (threadIdx.x < G) head[i * G + threadIdx.x] = sh.h[threadIdx.x];
-    if (threadIdx.x == 0) layer_score[i] = sh.J;
+    if (threadIdx.x == 0) layer_score[i] = sh.J - R;   // minimising: -(J of this layer) = J' - sum_g R_g
 }
 
 __global__ void chain_score_kernel(int Lyr, const int64_t* __restrict__ layer_score, ChainState* st, int64_t* J_q,
-                                   double* J, int32_t* iters_done) {
+                                   double* J, int32_t* iters_done, int minimize) {
     if (threadIdx.x != 0 || st->done) return;
     int64_t total = 0;
     for (int i = 0; i < Lyr; ++i) total += layer_score[i];
     st->iters += 1;
     *iters_done = st->iters;
-    *J_q = total;
-    *J = ldexp(static_cast<double>(total), -kNormBits);
+    const int64_t jq = minimize ? -total : total;
+    *J_q = jq;
+    *J = ldexp(static_cast<double>(jq), -kNormBits);
     if (total <= st->prev) st->done = 1;
     else st->prev = total;
+}
+
+// J of a given layout, per edge (Eq. objective): one block per edge, edge 2i =
+// up_i (h_i(g) == nu_i(k)), edge 2i+1 = down_i (nu_i(k) == h_{i+1}(g)).
+// Entries of h or nu outside [0, D) are reported as DTP_ERR_ARG.
+__global__ void __launch_bounds__(kThreads, 1)
+chain_edge_kernel(int Lyr, int G, int N, int D, const int64_t* __restrict__ nbuf, const int32_t* __restrict__ head,
+                  const int32_t* __restrict__ nu, int64_t* __restrict__ edge, ChainState* st, int* ws_status) {
+    __shared__ Shared sh;
+    if (*reinterpret_cast<volatile int*>(&st->done)) return;
+    const int e = blockIdx.x;
+    const int i = e >> 1;
+    const bool up = (e & 1) == 0;
+    const int64_t GN = static_cast<int64_t>(G) * N;
+    const int64_t* n = nbuf + (up ? i : Lyr + i) * GN;
+    const int32_t* hg = head + static_cast<int64_t>(up ? i : i + 1) * G;
+    const int32_t* nk = nu + static_cast<int64_t>(i) * N;
+    if (threadIdx.x < G) sh.h[threadIdx.x] = hg[threadIdx.x];
+    __syncthreads();
+    int bad = 0;
+    if (threadIdx.x < G && (sh.h[threadIdx.x] < 0 || sh.h[threadIdx.x] >= D)) bad = 1;
+    int64_t part = 0;
+    for (int k = threadIdx.x; k < N; k += kThreads) {
+        const int l = nk[k];
+        if (l < 0 || l >= D) {
+            bad = 1;
+            continue;
+        }
+        for (int g = 0; g < G; ++g)
+            if (sh.h[g] == l) part += n[static_cast<int64_t>(g) * N + k];
+    }
+    bad = __syncthreads_or(bad);
+    const int64_t tot = block_sum_i64(part, sh);
+    if (threadIdx.x == 0) {
+        edge[e] = tot;
+        if (bad) atomicMin(ws_status, static_cast<int>(DTP_ERR_ARG));
+    }
+}
+
+__global__ void chain_total_kernel(int n_edges, const int64_t* __restrict__ edge, const ChainState* st,
+                                   int64_t* J_q, double* J) {
+    if (threadIdx.x != 0 || st->done) return;
+    int64_t t = 0;
+    for (int e = 0; e < n_edges; ++e) t += edge[e];
+    *J_q = t;
+    *J = ldexp(static_cast<double>(t), -kNormBits);
 }
 
 // --------------------------------------------------------------------- host --
@@ -952,7 +1045,7 @@ static size_t chain_layout(int Lyr, int G, int N, int D, size_t* off_state, size
     *off_state = o;
     o += 256;
     *off_score = o;
-    o += align_up(static_cast<size_t>(Lyr) * sizeof(int64_t), 256);
+    o += align_up(static_cast<size_t>(2 * Lyr) * sizeof(int64_t), 256);   // layer scores / edge scores
     *off_prices = o;
     o += align_up(static_cast<size_t>(Lyr) * DMAX * sizeof(int64_t), 256);
     *off_nbuf = o;
@@ -968,7 +1061,8 @@ size_t chain_workspace_bytes(int Lyr, int G, int N, int D) {
 }
 
 template <int DT>
-static int launch_chain_t(const float* S_up, const float* S_down, int Lyr, int G, int N, int iters, int32_t* head,
+static int launch_chain_t(const float* S_up, const float* S_down, int Lyr, int G, int N, int iters,
+                          const uint8_t* move_heads, const uint8_t* move_neurons, int minimize, int32_t* head,
                           int32_t* nu, int64_t* J_q, double* J, int32_t* iters_done, uint8_t* ws,
                           cudaStream_t stream) {
     size_t o_state, o_score, o_prices, o_nbuf, o_gbuf;
@@ -986,32 +1080,60 @@ static int launch_chain_t(const float* S_up, const float* S_down, int Lyr, int G
     DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
     DTP_CUDA_TRY(cudaMemsetAsync(prices, 0, static_cast<size_t>(Lyr) * DMAX * sizeof(int64_t), stream));
     chain_init_kernel<<<1, 1, 0, stream>>>(st, J_q, J, iters_done);
-    chain_normalize_kernel<<<2 * Lyr - 1, kThreads, 0, stream>>>(S_up, S_down, Lyr, G, N, DT, nbuf, head, st,
+    chain_normalize_kernel<<<2 * Lyr - 1, kThreads, 0, stream>>>(S_up, S_down, Lyr, G, N, DT, nbuf, head, nu, st,
                                                                  ws_status);
     const uint32_t n_parts = static_cast<uint32_t>(partition_count(G, DT));
     for (int it = 0; it < iters; ++it) {
         chain_neuron_kernel<DT><<<Lyr, kThreads, dyn, stream>>>(Lyr, G, N, nbuf, head, nu, prices, st, ws_status, gbuf,
-                                                                 per_layer_bytes(N, DT), smem ? 1 : 0);
-        chain_head_kernel<DT><<<Lyr, kThreads, 0, stream>>>(Lyr, G, N, nbuf, nu, head, layer_score, st, n_parts);
-        chain_score_kernel<<<1, 32, 0, stream>>>(Lyr, layer_score, st, J_q, J, iters_done);
+                                                                 per_layer_bytes(N, DT), smem ? 1 : 0, move_neurons,
+                                                                 minimize);
+        chain_head_kernel<DT><<<Lyr, kThreads, 0, stream>>>(Lyr, G, N, nbuf, nu, head, layer_score, st, n_parts,
+                                                             move_heads, minimize);
+        chain_score_kernel<<<1, 32, 0, stream>>>(Lyr, layer_score, st, J_q, J, iters_done, minimize);
     }
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
 }
 
-int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters, int32_t* head,
-                 int32_t* nu, int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream) {
+int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters,
+                 const uint8_t* move_heads, const uint8_t* move_neurons, int minimize, int32_t* head, int32_t* nu,
+                 int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream) {
     uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+#define DTP_CHAIN_CASE(DV)                                                                                  \
+    case DV:                                                                                                \
+        return launch_chain_t<DV>(S_up, S_down, Lyr, G, N, iters, move_heads, move_neurons, minimize, head, nu, \
+                                  J_q, J, iters_done, ws, stream);
     switch (D) {
-        case 2: return launch_chain_t<2>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
-        case 3: return launch_chain_t<3>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
-        case 4: return launch_chain_t<4>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
-        case 5: return launch_chain_t<5>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
-        case 6: return launch_chain_t<6>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
-        case 7: return launch_chain_t<7>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
-        case 8: return launch_chain_t<8>(S_up, S_down, Lyr, G, N, iters, head, nu, J_q, J, iters_done, ws, stream);
+        DTP_CHAIN_CASE(2)
+        DTP_CHAIN_CASE(3)
+        DTP_CHAIN_CASE(4)
+        DTP_CHAIN_CASE(5)
+        DTP_CHAIN_CASE(6)
+        DTP_CHAIN_CASE(7)
+        DTP_CHAIN_CASE(8)
         default: return DTP_ERR_ARG;
     }
+#undef DTP_CHAIN_CASE
+}
+
+int launch_chain_score(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, const int32_t* head,
+                       const int32_t* nu, int64_t* edge_q, int64_t* J_q, double* J, void* workspace,
+                       cudaStream_t stream) {
+    uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+    size_t o_state, o_score, o_prices, o_nbuf, o_gbuf;
+    chain_layout(Lyr, G, N, D, &o_state, &o_score, &o_prices, &o_nbuf, &o_gbuf);
+    int* ws_status = reinterpret_cast<int*>(ws);
+    ChainState* st = reinterpret_cast<ChainState*>(ws + o_state);
+    int64_t* edge = edge_q ? edge_q : reinterpret_cast<int64_t*>(ws + o_score);
+    int64_t* nbuf = reinterpret_cast<int64_t*>(ws + o_nbuf);
+    DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
+    chain_init_kernel<<<1, 1, 0, stream>>>(st, J_q, J, nullptr);
+    chain_normalize_kernel<<<2 * Lyr - 1, kThreads, 0, stream>>>(S_up, S_down, Lyr, G, N, D, nbuf, nullptr, nullptr,
+                                                                 st, ws_status);
+    chain_edge_kernel<<<2 * Lyr - 1, kThreads, 0, stream>>>(Lyr, G, N, D, nbuf, head, nu, edge, st, ws_status);
+    chain_total_kernel<<<1, 32, 0, stream>>>(2 * Lyr - 1, edge, st, J_q, J);
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
 }
 
 }  // namespace search

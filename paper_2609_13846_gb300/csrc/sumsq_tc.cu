@@ -279,17 +279,19 @@ sumsq_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant_
 }
 
 // out[g, col] (+)= sum over row chunks (in order) of the unit partials; col < n_cols.
+// out row o sums groups o*qpg .. o*qpg + qpg - 1 (group by group, then row chunks).
 __global__ void sumsq_reduce_kernel(const float* __restrict__ partial, float* __restrict__ out, int groups,
-                                    int row_chunks, int col_tiles, int out_cols, int n_cols, int accumulate) {
-    const int64_t total = static_cast<int64_t>(groups) * n_cols;
+                                    int row_chunks, int col_tiles, int out_cols, int n_cols, int accumulate, int qpg) {
+    const int64_t total = static_cast<int64_t>(groups / qpg) * n_cols;
     for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
          idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int g = static_cast<int>(idx / n_cols);
+        const int o = static_cast<int>(idx / n_cols);
         const int col = static_cast<int>(idx % n_cols);
         const int j = col / out_cols, r = col % out_cols;
         float s = 0.0f;
-        for (int rc = 0; rc < row_chunks; ++rc)
-            s += partial[((static_cast<int64_t>(g) * row_chunks + rc) * col_tiles + j) * out_cols + r];
+        for (int g = o * qpg; g < (o + 1) * qpg; ++g)
+            for (int rc = 0; rc < row_chunks; ++rc)
+                s += partial[((static_cast<int64_t>(g) * row_chunks + rc) * col_tiles + j) * out_cols + r];
         out[idx] = accumulate ? out[idx] + s : s;
     }
 }
@@ -337,7 +339,7 @@ static bool map_bf16(CUtensorMap* m, const void* base, int rank, const cuuint64_
 
 template <int MODE>
 static int run(const CUtensorMap& ma, const CUtensorMap& mb0, const CUtensorMap& mb1, Params p, float* out,
-               int n_cols, int accumulate, cudaStream_t stream) {
+               int n_cols, int accumulate, cudaStream_t stream, int qpg = 1) {
     int dev = 0, sms = 0;
     DTP_CUDA_TRY(cudaGetDevice(&dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
@@ -346,10 +348,10 @@ static int run(const CUtensorMap& ma, const CUtensorMap& mb0, const CUtensorMap&
     const int grid = static_cast<int>(p.units < sms ? p.units : sms);
     sumsq_tc_kernel<MODE><<<grid, kThreads, kSmemBytes, stream>>>(ma, mb0, mb1, p);
     DTP_CUDA_TRY(cudaGetLastError());
-    const int64_t total = static_cast<int64_t>(p.groups) * n_cols;
+    const int64_t total = static_cast<int64_t>(p.groups / qpg) * n_cols;
     const int blocks = static_cast<int>((total + 255) / 256 < 4 * sms ? (total + 255) / 256 : 4 * sms);
     sumsq_reduce_kernel<<<blocks, 256, 0, stream>>>(p.partial, out, p.groups, p.row_chunks, p.col_tiles, p.out_cols,
-                                                    n_cols, accumulate);
+                                                    n_cols, accumulate, qpg);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
 }
@@ -401,8 +403,10 @@ size_t add_workspace_bytes(int64_t T, int G, int N) {
     return kWorkspaceHeader + static_cast<size_t>(units) * 128 * sizeof(float);
 }
 
-int launch_add(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
-               void* workspace, cudaStream_t stream) {
+// G heads of C; A_add receives G / qpg rows (qpg consecutive heads summed per row).
+int launch_add_grouped(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
+                       void* workspace, cudaStream_t stream, int qpg) {
+    if (qpg < 1 || G % qpg) return DTP_ERR_ARG;
     uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
     CUtensorMap mc, mg, mu;
     const cuuint64_t rs = static_cast<cuuint64_t>(d) * 2;
@@ -422,7 +426,12 @@ int launch_add(const void* C, const void* Wg, const void* Wu, int64_t T, int d, 
     p.out_cols = 128;
     p.partial = reinterpret_cast<float*>(ws + kWorkspaceHeader);
     p.status = reinterpret_cast<int*>(ws);
-    return run<kAdd>(mc, mg, mu, p, A_add, N, 1, stream);
+    return run<kAdd>(mc, mg, mu, p, A_add, N, 1, stream, qpg);
+}
+
+int launch_add(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
+               void* workspace, cudaStream_t stream) {
+    return launch_add_grouped(C, Wg, Wu, T, d, G, N, A_add, workspace, stream, 1);
 }
 
 }  // namespace sq

@@ -58,6 +58,12 @@ def lib():
     L.dtp_affinity_accumulate_noalloc.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp]
     L.dtp_affinity_accumulate_ex.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _vp,
                                              _sz, _vp]
+    L.dtp_affinity_grouped_workspace_size.argtypes = [_i64, _i32, _i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_affinity_accumulate_grouped.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _i32, _vp,
+                                                  _vp, _vp, _sz, _vp]
+    L.dtp_affinity_add_grouped_workspace_size.argtypes = [_i64, _i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_affinity_add_accumulate_grouped.argtypes = [_vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _sz,
+                                                      _vp]
     L.dtp_affinity_add_workspace_size.argtypes = [_i64, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_affinity_add_accumulate.argtypes = [_vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
     L.dtp_down_weight_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
@@ -65,12 +71,18 @@ def lib():
     L.dtp_down_finalize.argtypes = [_vp, _vp, _i32, _i32, _i64, _vp, _vp]
     L.dtp_search_chain_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_chain.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+    L.dtp_search_chain_ex.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp,
+                                      _vp, _vp, _sz, _vp]
+    L.dtp_chain_score.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_search_layout_batched.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                             _vp]
-    for fn in ("dtp_search_chain_workspace_size", "dtp_search_chain", "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
+    for fn in ("dtp_search_chain_workspace_size", "dtp_search_chain", "dtp_search_chain_ex", "dtp_chain_score",
+               "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
+               "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
+               "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
                "dtp_down_weight_workspace_size", "dtp_down_weight_sqnorm", "dtp_down_finalize",
                "dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
                "dtp_affinity_finalize",
@@ -93,6 +105,22 @@ def _check(fn: str, status: int):
 def _stream(stream=None) -> int:
     s = torch.cuda.current_stream() if stream is None else stream
     return int(s.cuda_stream)
+
+
+def _keep(t: torch.Tensor, stream) -> torch.Tensor:
+    """Mark a temporary as in use on ``stream`` so the caching allocator does not hand it out early."""
+    if stream is not None:
+        t.record_stream(stream)
+    return t
+
+
+def _device_mask(m, L: int, dev, stream) -> torch.Tensor | None:
+    if m is None:
+        return None
+    t = torch.as_tensor(m).reshape(-1)
+    if t.numel() != L:
+        raise ValueError(f"layer mask must have {L} entries, got {t.numel()}")
+    return _keep((t != 0).to(torch.uint8).to(dev).contiguous(), stream)
 
 
 def _ptr(t: torch.Tensor | None):
@@ -175,6 +203,76 @@ def affinity_accumulate_down(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Ten
                                           _stream(stream))
     _check("dtp_affinity_accumulate_ex", st)
     return A, act2
+
+
+def affinity_grouped_workspace_size(T: int, d: int, H_q: int, q_per_group: int, N: int, dtype: int) -> int:
+    n = _sz(0)
+    _check("dtp_affinity_grouped_workspace_size",
+           lib().dtp_affinity_grouped_workspace_size(T, d, H_q, q_per_group, N, dtype, ctypes.byref(n)))
+    return n.value
+
+
+def affinity_accumulate_grouped(X: torch.Tensor, C_q: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
+                                q_per_group: int, A: torch.Tensor | None = None, rms_next: torch.Tensor | None = None,
+                                act2: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                                stream=None):
+    """First-order score per query head, summed over each KV group's query heads (Sec. 3).
+
+    C_q [H_q, T, d] holds each query head's write; A [H_q / q_per_group, N] fp32
+    is accumulated into.  With rms_next [T] the down-edge activation term is
+    added to act2 [N] as in affinity_accumulate_down.  Returns A, or (A, act2)
+    when rms_next is given.
+    """
+    for name, t in (("X", X), ("C_q", C_q), ("W_gate", W_gate), ("W_up", W_up)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    if not (X.dtype == C_q.dtype == W_gate.dtype == W_up.dtype):
+        raise TypeError("X, C_q, W_gate and W_up must share one dtype")
+    T, d = X.shape
+    Hq = C_q.shape[0]
+    N = W_gate.shape[0]
+    if C_q.shape != (Hq, T, d) or W_gate.shape != (N, d) or W_up.shape != (N, d):
+        raise ValueError("shapes must be X [T,d], C_q [H_q,T,d], W_gate [N,d], W_up [N,d]")
+    if q_per_group < 1 or Hq % q_per_group:
+        raise ValueError("q_per_group must divide H_q")
+    code = _dtype_code(X)
+    if A is None:
+        A = torch.zeros((Hq // q_per_group, N), dtype=torch.float32, device=X.device)
+    if rms_next is not None:
+        if rms_next.shape != (T,) or rms_next.dtype != torch.float32:
+            raise ValueError("rms_next must be fp32 [T]")
+        if act2 is None:
+            act2 = torch.zeros(N, dtype=torch.float32, device=X.device)
+    if workspace is None:
+        workspace = _keep(torch.empty(affinity_grouped_workspace_size(T, d, Hq, q_per_group, N, code),
+                                      dtype=torch.uint8, device=X.device), stream)
+    st = lib().dtp_affinity_accumulate_grouped(_ptr(X), _ptr(C_q), _ptr(W_gate), _ptr(W_up), _ptr(rms_next), T, d,
+                                               Hq, q_per_group, N, code, _ptr(A),
+                                               _ptr(act2) if rms_next is not None else None, _ptr(workspace),
+                                               workspace.numel(), _stream(stream))
+    _check("dtp_affinity_accumulate_grouped", st)
+    return (A, act2) if rms_next is not None else A
+
+
+def affinity_add_accumulate_grouped(C_q: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor, q_per_group: int,
+                                    A_add: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                                    stream=None) -> torch.Tensor:
+    """ADD score per query head, summed over each KV group's query heads (Sec. 3); bf16 inputs."""
+    Hq, T, d = C_q.shape
+    N = W_gate.shape[0]
+    if q_per_group < 1 or Hq % q_per_group:
+        raise ValueError("q_per_group must divide H_q")
+    if A_add is None:
+        A_add = torch.zeros((Hq // q_per_group, N), dtype=torch.float32, device=C_q.device)
+    if workspace is None:
+        n = _sz(0)
+        _check("dtp_affinity_add_grouped_workspace_size",
+               lib().dtp_affinity_add_grouped_workspace_size(T, d, Hq, q_per_group, N, ctypes.byref(n)))
+        workspace = _keep(torch.empty(n.value, dtype=torch.uint8, device=C_q.device), stream)
+    st = lib().dtp_affinity_add_accumulate_grouped(_ptr(C_q), _ptr(W_gate), _ptr(W_up), T, d, Hq, q_per_group, N,
+                                                   _ptr(A_add), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_affinity_add_accumulate_grouped", st)
+    return A_add
 
 
 def affinity_add_accumulate(C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
@@ -310,33 +408,82 @@ def search_layout(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor |
     return {k: v[0] for k, v in r.items()}
 
 
-def search_chain(S_up: torch.Tensor, S_down: torch.Tensor | None, D: int, iters: int,
-                 workspace: torch.Tensor | None = None, stream=None, check: bool = True) -> dict:
-    """Coordinate ascent on the whole-model objective (Sec. 3, Eq. objective, up and down edges).
-
-    S_up [L, H_kv, N], S_down [L-1, H_kv, N] (None when L == 1), fp32 CUDA.
-    Returns device tensors: h [L,H_kv] int32, nu [L,N] int32, J_q int64 (units
-    of 2^-43), J float64, iters_done int32.  Asynchronous unless ``check``.
-    """
+def _chain_inputs(S_up: torch.Tensor, S_down: torch.Tensor | None):
     if S_up.dtype != torch.float32 or not S_up.is_cuda or not S_up.is_contiguous():
         raise ValueError("S_up must be a contiguous fp32 CUDA tensor [L, H_kv, N]")
     Lyr, H, N = S_up.shape
-    if Lyr > 1 and (S_down is None or S_down.shape != (Lyr - 1, H, N) or not S_down.is_contiguous()):
-        raise ValueError("S_down must be a contiguous fp32 tensor [L-1, H_kv, N]")
+    if Lyr > 1 and (S_down is None or S_down.shape != (Lyr - 1, H, N) or not S_down.is_contiguous()
+                    or S_down.dtype != torch.float32 or S_down.device != S_up.device):
+        raise ValueError("S_down must be a contiguous fp32 tensor [L-1, H_kv, N] on S_up's device")
+    return Lyr, H, N
+
+
+def search_chain_workspace_size(layers: int, H_kv: int, N: int, D: int) -> int:
+    """Bytes of workspace for search_chain and chain_score."""
+    n = _sz(0)
+    _check("dtp_search_chain_workspace_size",
+           lib().dtp_search_chain_workspace_size(layers, H_kv, N, D, ctypes.byref(n)))
+    return n.value
+
+
+def _chain_workspace(Lyr, H, N, D, dev, stream):
+    return _keep(torch.empty(search_chain_workspace_size(Lyr, H, N, D), dtype=torch.uint8, device=dev), stream)
+
+
+def search_chain(S_up: torch.Tensor, S_down: torch.Tensor | None, D: int, iters: int,
+                 workspace: torch.Tensor | None = None, stream=None, check: bool = True,
+                 move_heads=None, move_neurons=None, minimize: bool = False) -> dict:
+    """Coordinate ascent on the whole-model objective (Sec. 3, Eq. objective, up and down edges).
+
+    S_up [L, H_kv, N], S_down [L-1, H_kv, N] (None when L == 1), fp32 CUDA.
+    move_heads / move_neurons: per-layer 0/1 (None = every layer moves) and
+    minimize: the ablation layouts of Sec. 3 'Optimiser' (Table 4).
+    Returns device tensors: h [L,H_kv] int32, nu [L,N] int32, J_q int64 (units
+    of 2^-43), J float64, iters_done int32.  Asynchronous unless ``check``.
+    """
+    Lyr, H, N = _chain_inputs(S_up, S_down)
     dev = S_up.device
     out = dict(h=torch.empty((Lyr, H), dtype=torch.int32, device=dev),
                nu=torch.empty((Lyr, N), dtype=torch.int32, device=dev),
                J_q=torch.empty((), dtype=torch.int64, device=dev),
                J=torch.empty((), dtype=torch.float64, device=dev),
                iters_done=torch.empty((), dtype=torch.int32, device=dev))
+    mh = _device_mask(move_heads, Lyr, dev, stream)
+    mn = _device_mask(move_neurons, Lyr, dev, stream)
     if workspace is None:
-        n = _sz(0)
-        _check("dtp_search_chain_workspace_size", lib().dtp_search_chain_workspace_size(Lyr, H, N, D, ctypes.byref(n)))
-        workspace = torch.empty(n.value, dtype=torch.uint8, device=dev)
-    st = lib().dtp_search_chain(_ptr(S_up), _ptr(S_down) if Lyr > 1 else None, Lyr, H, N, D, iters, _ptr(out["h"]),
-                                _ptr(out["nu"]), _ptr(out["J_q"]), _ptr(out["J"]), _ptr(out["iters_done"]),
-                                _ptr(workspace), workspace.numel(), _stream(stream))
-    _check("dtp_search_chain", st)
+        workspace = _chain_workspace(Lyr, H, N, D, dev, stream)
+    st = lib().dtp_search_chain_ex(_ptr(S_up), _ptr(S_down) if Lyr > 1 else None, Lyr, H, N, D, iters, _ptr(mh),
+                                   _ptr(mn), int(bool(minimize)), _ptr(out["h"]), _ptr(out["nu"]), _ptr(out["J_q"]),
+                                   _ptr(out["J"]), _ptr(out["iters_done"]), _ptr(workspace), workspace.numel(),
+                                   _stream(stream))
+    _check("dtp_search_chain_ex", st)
     if check:
-        _check("dtp_search_chain (device status)", workspace_status(workspace, stream))
+        _check("dtp_search_chain_ex (device status)", workspace_status(workspace, stream))
+    return out
+
+
+def chain_score(S_up: torch.Tensor, S_down: torch.Tensor | None, h: torch.Tensor, nu: torch.Tensor, D: int,
+                workspace: torch.Tensor | None = None, stream=None, check: bool = True) -> dict:
+    """J of a given layout (Eq. objective) and its per-edge terms.
+
+    h [L, H_kv], nu [L, N] int32 CUDA, entries in [0, D).  Returns device
+    tensors: edge_q [2L-1] int64 (up_0, down_0, up_1, ...; units of 2^-43 of
+    each edge), J_q int64, J float64.
+    """
+    Lyr, H, N = _chain_inputs(S_up, S_down)
+    dev = S_up.device
+    for name, t, shape in (("h", h, (Lyr, H)), ("nu", nu, (Lyr, N))):
+        if t.dtype != torch.int32 or t.device != dev or not t.is_contiguous() or tuple(t.shape) != shape:
+            raise ValueError(f"{name} must be a contiguous int32 tensor {shape} on S_up's device")
+    out = dict(edge_q=torch.empty(2 * Lyr - 1, dtype=torch.int64, device=dev),
+               J_q=torch.empty((), dtype=torch.int64, device=dev),
+               J=torch.empty((), dtype=torch.float64, device=dev))
+    if workspace is None:
+        workspace = _chain_workspace(Lyr, H, N, D, dev, stream)
+    st = lib().dtp_chain_score(_ptr(S_up), _ptr(S_down) if Lyr > 1 else None, Lyr, H, N, D, _ptr(h), _ptr(nu),
+                               _ptr(out["edge_q"]), _ptr(out["J_q"]), _ptr(out["J"]), _ptr(workspace),
+                               workspace.numel(), _stream(stream))
+    _check("dtp_chain_score", st)
+    if check:
+        _check("dtp_chain_score (device status)", workspace_status(workspace, stream))
     return out

@@ -98,3 +98,40 @@ def test_search_rejects_missing_workspace(lib):
     vp = ctypes.c_void_p
     ok = vp(1 << 20)
     assert lib.dtp_search_layout(ok, 8, 64, 2, 3, ok, ok, ok, ok, ok, None, 0, None) == -5
+
+
+@pytest.mark.parametrize("args,ok", [
+    ((16384, 1024, 16, 2, 3072, 0), True), ((16, 64, 32, 4, 128, 0), True), ((16, 64, 128, 16, 128, 1), True),
+    ((16, 64, 34, 2, 128, 0), False),        # 17 KV groups
+    ((16, 64, 16, 3, 128, 0), False),        # q_per_group does not divide H_q
+    ((16, 64, 136, 8, 128, 0), False),       # more than 128 query heads
+    ((16, 64, 16, 0, 128, 0), False), ((16, 12, 16, 2, 128, 0), False)])
+def test_grouped_size_queries(lib, args, ok):
+    n = ctypes.c_size_t(0)
+    st = lib.dtp_affinity_grouped_workspace_size(*args, ctypes.byref(n))
+    assert (st == 0) == ok
+    T, d, Hq, q, N, dtype = args
+    st2 = lib.dtp_affinity_add_grouped_workspace_size(T, d, Hq, q, N, ctypes.byref(n))
+    assert (st2 == 0) == ok
+
+
+def test_grouped_workspace_covers_one_launch_of_whole_groups(lib):
+    from paper_2609_13846_gb300 import dtp
+    # 32 query heads at 4 per group run as two launches of 16 heads: the workspace of one 16-head launch
+    assert dtp.affinity_grouped_workspace_size(4096, 1024, 32, 4, 3072, dtp.DTP_BF16) == \
+        dtp.affinity_workspace_size(4096, 1024, 16, 3072, dtp.DTP_BF16)
+    # 6 heads at 3 per group: one launch of all 6
+    assert dtp.affinity_grouped_workspace_size(300, 64, 6, 3, 130, dtp.DTP_F32) == \
+        dtp.affinity_workspace_size(300, 64, 6, 130, dtp.DTP_F32)
+
+
+def test_chain_score_and_ablation_reject_before_launch(lib):
+    buf = ctypes.create_string_buffer(1 << 16)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    # bad sizes (D does not divide N)
+    assert lib.dtp_chain_score(p, p, 2, 8, 30, 4, p, p, None, p, p, p, ctypes.c_size_t(1 << 16), None) == -1
+    # missing outputs
+    assert lib.dtp_search_chain_ex(p, p, 2, 8, 32, 4, 5, None, None, 1, None, p, p, p, p, p,
+                                   ctypes.c_size_t(1 << 16), None) == -1
+    # too small a workspace
+    assert lib.dtp_chain_score(p, p, 2, 8, 32, 4, p, p, None, p, p, p, ctypes.c_size_t(16), None) == -5

@@ -83,3 +83,73 @@ def test_chain_invalid_entry_reported():
     with pytest.raises(dtp.DTPError) as e:
         dtp.search_chain(torch.as_tensor(Su, device=DEV), torch.as_tensor(Sd, device=DEV), 2, 10)
     assert e.value.status == dtp.DTP_ERR_ARG
+
+
+# ------------------------------------------------------------- ablations ----
+
+from paper_2609_13846_gb300 import ablation  # noqa: E402
+
+
+def _compare_ablation(Su, Sd, D, iters, kind):
+    Lyr = Su.shape[0]
+    mh, mn, mini = ablation.ablation_masks(Lyr, kind)
+    gSu = torch.as_tensor(Su, device=DEV).contiguous()
+    gSd = torch.as_tensor(Sd, device=DEV).contiguous() if Lyr > 1 else None
+    res = dtp.search_chain(gSu, gSd, D, iters, move_heads=mh, move_neurons=mn, minimize=mini)
+    ref = oracle.chain_search(Su, Sd if Lyr > 1 else None, D, iters, move_heads=mh, move_neurons=mn, minimize=mini)
+    np.testing.assert_array_equal(res["h"].cpu().numpy(), ref["h"])
+    np.testing.assert_array_equal(res["nu"].cpu().numpy(), ref["nu"])
+    assert int(res["J_q"]) == ref["J_q"]
+    assert int(res["iters_done"]) == ref["iters_done"]
+    assert float(res["J"]) == ref["J"]
+    return ref
+
+
+@pytest.mark.parametrize("kind", ["anti", "heads_only", "neurons_only", "layers2", "layers3"])
+@pytest.mark.parametrize("L,G,N,D", [(6, 8, 256, 2), (6, 8, 512, 4), (3, 6, 96, 3), (4, 8, 64, 8), (1, 8, 128, 4)])
+def test_chain_ablations_match_oracle(kind, L, G, N, D):
+    if kind.startswith("layers") and int(kind[6:]) > L:
+        pytest.skip("subset larger than the model")
+    Su, Sd = _model(L, G, N, seed=7 * L + N + D)
+    _compare_ablation(Su, Sd, D, 10, kind)
+
+
+@pytest.mark.parametrize("kind", ["anti", "neurons_only", "layers4"])
+def test_chain_ablations_qwen_shaped(kind):
+    """28 layers x (G=8, N=3072) at D=4: the Table 4 ablations, bit-exact."""
+    Su, Sd = _model(28, 8, 3072, seed=100)
+    _compare_ablation(Su, Sd, 4, 10, kind)
+
+
+def test_chain_anti_on_integer_ties():
+    """Integer-valued affinities leave many equal gains; minimising must pick the same canonical layout."""
+    Su, Sd = _model(5, 8, 256, seed=3, kind="integer")
+    for D in (2, 4):
+        _compare_ablation(Su, Sd, D, 10, "anti")
+
+
+@pytest.mark.parametrize("L,G,N,D", [(1, 8, 256, 2), (5, 8, 384, 4), (28, 8, 3072, 4), (3, 6, 96, 3)])
+def test_chain_score_matches_oracle(L, G, N, D):
+    Su, Sd = _model(L, G, N, seed=L + N)
+    gSu = torch.as_tensor(Su, device=DEV).contiguous()
+    gSd = torch.as_tensor(Sd, device=DEV).contiguous() if L > 1 else None
+    for seed in (1000, 1001, 1002):
+        h, nu = ablation.random_layout(L, G, N, D, seed)
+        r = dtp.chain_score(gSu, gSd, torch.as_tensor(h, device=DEV), torch.as_tensor(nu, device=DEV), D)
+        ref_e = oracle.chain_edge_scores(Su, Sd if L > 1 else None, h, nu)
+        np.testing.assert_array_equal(r["edge_q"].cpu().numpy(), ref_e)
+        assert int(r["J_q"]) == int(ref_e.sum()) == oracle.chain_score(Su, Sd if L > 1 else None, h, nu)
+    # the optimiser's own layout scores its own J
+    res = dtp.search_chain(gSu, gSd, D, 10)
+    r = dtp.chain_score(gSu, gSd, res["h"], res["nu"], D)
+    assert int(r["J_q"]) == int(res["J_q"])
+
+
+def test_chain_score_rejects_out_of_range_layout():
+    Su, Sd = _model(3, 8, 64, seed=5)
+    h, nu = ablation.random_layout(3, 8, 64, 4, 1000)
+    nu[1, 7] = 4
+    with pytest.raises(dtp.DTPError) as e:
+        dtp.chain_score(torch.as_tensor(Su, device=DEV), torch.as_tensor(Sd, device=DEV),
+                        torch.as_tensor(h, device=DEV), torch.as_tensor(nu, device=DEV), 4)
+    assert e.value.status == dtp.DTP_ERR_ARG
