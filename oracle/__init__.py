@@ -70,6 +70,11 @@ def _load():
     lib.oracle_search_layout.argtypes = [_f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                          _i32p, _i32p, _i64p, _f64p, _i32p, _i32p]
     lib.oracle_search_layout.restype = ctypes.c_int
+    lib.oracle_head_writes.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
+                                       ctypes.c_int, ctypes.c_int, _f64p]
+    lib.oracle_head_writes.restype = None
+    lib.oracle_layout_order.argtypes = [_i32p, ctypes.c_int, ctypes.c_int, _i32p]
+    lib.oracle_layout_order.restype = ctypes.c_int
     lib.oracle_hungarian_max.argtypes = [_i64p, ctypes.c_int, _i32p]
     lib.oracle_hungarian_max.restype = ctypes.c_int64
     lib.oracle_affinity_add.argtypes = [_f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
@@ -357,4 +362,36 @@ def chain_edge_scores(S_up, S_down, h, nu) -> np.ndarray:
                                            _p(_c(nu, np.int32), _i32p), _p(out, _i64p))
     if bad:
         raise ValueError("negative or non-finite affinity entry")
+    return out
+
+
+def head_writes(attn, W_o, gamma, rms, head_dim: int, q_per_row: int = 1) -> np.ndarray:
+    """p_h = gamma . (a_h W_o^(h)T) / r per head (Sec. 3), rows summed over q_per_row consecutive heads.
+
+    attn [T, Hq*hd], W_o [d, Hq*hd], gamma [d], rms [T]; returns C [Hq/q_per_row, T, d] fp64.
+    """
+    A = _c(attn, np.float64)
+    W = _c(W_o, np.float64)
+    g = _c(gamma, np.float64)
+    r = _c(rms, np.float64)
+    T, K = A.shape
+    d = W.shape[0]
+    if K % head_dim or W.shape != (d, K) or g.shape != (d,) or r.shape != (T,):
+        raise ValueError("shapes must be attn [T, Hq*hd], W_o [d, Hq*hd], gamma [d], rms [T]")
+    Hq = K // head_dim
+    if q_per_row < 1 or Hq % q_per_row:
+        raise ValueError("q_per_row must divide the number of heads")
+    C = np.zeros((Hq // q_per_row, T, d), np.float64)
+    _load().oracle_head_writes(_p(A, _f64p), _p(W, _f64p), _p(g, _f64p), _p(r, _f64p), T, d, Hq, head_dim,
+                               q_per_row, _p(C, _f64p))
+    return C
+
+
+def layout_order(labels, D: int) -> np.ndarray:
+    """Items listed device by device (each device's in increasing index): the permutation that
+    makes every device's items one contiguous shard."""
+    lab = _c(labels, np.int32)
+    out = np.zeros(lab.shape[0], np.int32)
+    if _load().oracle_layout_order(_p(lab, _i32p), lab.shape[0], D, _p(out, _i32p)) != 0:
+        raise ValueError("label outside [0, D)")
     return out

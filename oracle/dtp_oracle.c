@@ -31,6 +31,10 @@
  *   oracle_normalize_unit_mass, oracle_chain_search
  *                          Sec. 3 "Objective" (Eq. objective, both sums) and
  *                          "Optimiser" over all layers of a model.
+ *   oracle_head_writes     Sec. 3 "Affinity scores": head h's write into the
+ *                          FFN input, p_h = gamma . (a_h W_o^(h)) / r.
+ *   oracle_layout_order    Sec. 3 (sharding a permuted dense model): the
+ *                          order that groups heads / neurons by device.
  *
  * Nothing here is shared with the CUDA library: no header, table or helper.
  * Only the tests, the smoke check and the benchmark's CPU-baseline leg load
@@ -782,6 +786,50 @@ int oracle_chain_edge_scores(const float* S_up, const float* S_down, int L, int 
     }
     free(n);
     return bad;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Producer and layout application                                           */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Head writes into the FFN input (Sec. 3): attention head h's output a_h
+ * (columns h*hd .. h*hd+hd-1 of attn [T, Hq*hd]) enters the residual as
+ * a_h W_o^(h)T (the matching columns of W_o [d, Hq*hd]), and reaches the FFN
+ * input through its pre-norm as gamma . (a_h W_o^(h)T) / r with r the rms of
+ * the residual at that token (held fixed).  Row j of C sums the q_per_row
+ * consecutive heads j*q_per_row ..; q_per_row = 1 gives one row per query
+ * head, q_per_row = query heads per KV group gives the group's write.
+ *   C [Hq/q_per_row, T, d] fp64, overwritten.
+ */
+void oracle_head_writes(const double* attn, const double* Wo, const double* gamma, const double* rms, int64_t T,
+                        int d, int Hq, int hd, int q_per_row, double* C) {
+    const int K = Hq * hd, rows = Hq / q_per_row, Kj = q_per_row * hd;
+    #pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < T; ++t)
+        for (int j = 0; j < rows; ++j)
+            for (int i = 0; i < d; ++i) {
+                double s = 0.0;
+                for (int c = j * Kj; c < (j + 1) * Kj; ++c) s += attn[t * K + c] * Wo[(int64_t)i * K + c];
+                C[((int64_t)j * T + t) * d + i] = gamma[i] * s / rms[t];
+            }
+}
+
+/*
+ * The order that groups items by device: order[p] = the item at position p
+ * when items are listed device by device, each device's items in increasing
+ * index.  For a balanced layout, positions p*D/n .. of the permuted model are
+ * device floor(p D / n)'s contiguous shard.  Returns OR_ERR_ARG on a label
+ * outside [0, D).
+ */
+int oracle_layout_order(const int* labels, int n, int D, int* order) {
+    for (int k = 0; k < n; ++k)
+        if (labels[k] < 0 || labels[k] >= D) return OR_ERR_ARG;
+    int pos = 0;
+    for (int l = 0; l < D; ++l)
+        for (int k = 0; k < n; ++k)
+            if (labels[k] == l) order[pos++] = k;
+    return OR_OK;
 }
 
 /* ------------------------------------------------------------------------ */
