@@ -377,6 +377,68 @@ int dtp_chain_score(const float* S_up, const float* S_down, int layers, int H_kv
                     const int32_t* head_part, const int32_t* neuron_dev, int64_t* edge_q, int64_t* J_q, double* J,
                     void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * The producer of C (Sec. 3, "Affinity scores"): each attention head's write
+ * into the FFN input, with the rms held fixed,
+ *     C[j, t, :] = gamma . ( sum over heads h of row j of a_{h,t} W_o^(h)T ) / rms[t]
+ *   attn   [T, H_q*head_dim] bf16, device: the heads' outputs before o_proj
+ *          (head h in columns h*head_dim .. h*head_dim + head_dim - 1)
+ *   W_o    [d, H_q*head_dim] bf16, device: o_proj (nn.Linear [out, in])
+ *   gamma  [d] fp32, device, 16-byte aligned: the FFN pre-norm gain
+ *   rms    [T] fp32, device, > 0: rms of the residual entering that norm
+ *   q_per_row  heads per output row: 1 = one row per query head (for
+ *          dtp_affinity_accumulate_grouped), query heads per KV group = the
+ *          group's combined write (for dtp_affinity_accumulate)
+ *   C      [H_q / q_per_row, T, d] bf16 out, device (rounded once, RN)
+ * head_dim a multiple of 16; d a multiple of 8; H_q * head_dim <= 2^20.
+ * tcgen05 GEMM with fp32 accumulation; the fp32 product is scaled by
+ * gamma / rms before the rounding.  Workspace: dtp_head_writes_workspace_size
+ * bytes (a status word).  Asynchronous; T == 0 returns DTP_OK.
+ */
+int dtp_head_writes_workspace_size(size_t* bytes);
+int dtp_head_writes(const void* attn, const void* W_o, const float* gamma, const float* rms, int64_t T, int d,
+                    int H_q, int head_dim, int q_per_row, void* C, void* workspace, size_t workspace_bytes,
+                    void* stream);
+
+/*
+ * Applying a layout to the dense weights (Sec. 3: the permuted dense model is
+ * sharded into contiguous slices).  dtp_layout_order turns device labels into
+ * the order that lists every device's items contiguously:
+ *     order[i][p] = the item at position p when layer i's items are listed
+ *                   device by device, each device's in increasing index
+ *   labels  [layers, n] int32, device: head_part or neuron_dev
+ *   order   [layers, n] int32 out, device
+ *   balanced  nonzero: also require n / D items per device, so that position
+ *             p belongs to device floor(p D / n)
+ * Labels outside [0, D), or an unbalanced layer when `balanced`, are reported
+ * as DTP_ERR_ARG through the workspace status word (order undefined).
+ * Workspace: dtp_head_writes_workspace_size bytes.  Asynchronous.
+ */
+int dtp_layout_order(const int32_t* labels, int layers, int n, int D, int balanced, int32_t* order,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Gathers that apply the order to weights stored [layers, rows, ...]
+ * contiguous (one matrix per layer, back to back), src and dst distinct:
+ *   dtp_permute_rows: dst[i][b*block_rows + r][:] = src[i][perm[i][b]*block_rows + r][:]
+ *     rows of row_bytes bytes; q_proj (block = query heads per group *
+ *     head_dim rows per KV group), k_proj / v_proj (block = head_dim),
+ *     gate_proj / up_proj (block = 1 row per neuron)
+ *   dtp_permute_cols: dst[i][r][b*block_cols + c] = src[i][r][perm[i][b]*block_cols + c]
+ *     elements of elem_bytes bytes; o_proj (block = query heads per group *
+ *     head_dim columns), down_proj (block = 1 column per neuron)
+ *   perm  int32, device, layer i's entries at perm + i * perm_layer_stride
+ * An entry of perm outside [0, blocks) is not followed: the affected elements
+ * are left unwritten and DTP_ERR_ARG is reported through the workspace status
+ * word.  Workspace: dtp_head_writes_workspace_size bytes.  Asynchronous.
+ */
+int dtp_permute_rows(const void* src, void* dst, int layers, int64_t rows, int64_t row_bytes, int block_rows,
+                     const int32_t* perm, int64_t perm_layer_stride, void* workspace, size_t workspace_bytes,
+                     void* stream);
+int dtp_permute_cols(const void* src, void* dst, int layers, int64_t rows, int64_t cols, int elem_bytes,
+                     int block_cols, const int32_t* perm, int64_t perm_layer_stride, void* workspace,
+                     size_t workspace_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -31,6 +31,18 @@ int launch_add(const void* C, const void* Wg, const void* Wu, int64_t T, int d, 
 int launch_add_grouped(const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A_add,
                        void* workspace, cudaStream_t stream, int qpg);
 }  // namespace sq
+namespace hw {
+int launch(const void* attn, const void* Wo, const float* gamma, const float* rms, int64_t T, int d, int Hq, int hd,
+           int q_per_row, void* C, void* workspace, cudaStream_t stream);
+}  // namespace hw
+namespace apply {
+int launch_order(const int32_t* labels, int layers, int n, int D, int balanced, int32_t* order, void* workspace,
+                 cudaStream_t stream);
+int launch_rows(const void* src, void* dst, int layers, int64_t rows, int64_t row_bytes, int block_rows,
+                const int32_t* perm, int64_t perm_stride, void* workspace, cudaStream_t stream);
+int launch_cols(const void* src, void* dst, int layers, int64_t rows, int64_t row_bytes, int64_t block_bytes,
+                int elem_bytes, const int32_t* perm, int64_t perm_stride, void* workspace, cudaStream_t stream);
+}  // namespace apply
 int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream);
 int launch_down_finalize(const float* act2, const float* bn, int G, int N, int64_t T_total, float* S,
                          cudaStream_t stream);
@@ -230,6 +242,67 @@ int dtp_affinity_add_accumulate_grouped(const void* C_q, const void* W_gate, con
         if (st != DTP_OK) return st;
     }
     return DTP_OK;
+}
+
+int dtp_head_writes_workspace_size(size_t* bytes) {
+    if (!bytes) return DTP_ERR_ARG;
+    *bytes = kWorkspaceHeader;
+    return DTP_OK;
+}
+
+int dtp_head_writes(const void* attn, const void* W_o, const float* gamma, const float* rms, int64_t T, int d,
+                    int H_q, int head_dim, int q_per_row, void* C, void* workspace, size_t workspace_bytes,
+                    void* stream) {
+    if (T < 0 || T > (int64_t(1) << 31) - 256 || d < 8 || d % 8 || H_q < 1 || head_dim < 16 || head_dim % 16 ||
+        q_per_row < 1 || H_q % q_per_row || static_cast<int64_t>(H_q) * head_dim > (int64_t(1) << 20) ||
+        H_q / q_per_row > 65535)
+        return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;
+    if (!attn || !W_o || !gamma || !rms || !C || !aligned16(attn) || !aligned16(W_o) || !aligned16(gamma) ||
+        !aligned16(C) || (reinterpret_cast<uintptr_t>(rms) & 3))
+        return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < kWorkspaceHeader || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    return hw::launch(attn, W_o, gamma, rms, T, d, H_q, head_dim, q_per_row, C, workspace, s);
+}
+
+int dtp_layout_order(const int32_t* labels, int layers, int n, int D, int balanced, int32_t* order, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+    if (layers < 1 || layers > 65535 || n < 1 || D < 1 || D > n || (balanced && n % D)) return DTP_ERR_ARG;
+    if (!labels || !order || (reinterpret_cast<uintptr_t>(labels) & 3) || (reinterpret_cast<uintptr_t>(order) & 3))
+        return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < kWorkspaceHeader || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    return apply::launch_order(labels, layers, n, D, balanced ? 1 : 0, order, workspace, s);
+}
+
+int dtp_permute_rows(const void* src, void* dst, int layers, int64_t rows, int64_t row_bytes, int block_rows,
+                     const int32_t* perm, int64_t perm_layer_stride, void* workspace, size_t workspace_bytes,
+                     void* stream) {
+    if (layers < 1 || rows < 1 || row_bytes < 1 || block_rows < 1 || rows % block_rows ||
+        perm_layer_stride < rows / block_rows)
+        return DTP_ERR_ARG;
+    if (!src || !dst || !perm || src == dst || (reinterpret_cast<uintptr_t>(perm) & 3)) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < kWorkspaceHeader || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    return apply::launch_rows(src, dst, layers, rows, row_bytes, block_rows, perm, perm_layer_stride, workspace, s);
+}
+
+int dtp_permute_cols(const void* src, void* dst, int layers, int64_t rows, int64_t cols, int elem_bytes,
+                     int block_cols, const int32_t* perm, int64_t perm_layer_stride, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+    if (layers < 1 || rows < 1 || cols < 1 || elem_bytes < 1 || elem_bytes > 16 || block_cols < 1 ||
+        cols % block_cols || perm_layer_stride < cols / block_cols || cols * elem_bytes >= (int64_t(1) << 31))
+        return DTP_ERR_ARG;
+    if (!src || !dst || !perm || src == dst || (reinterpret_cast<uintptr_t>(perm) & 3)) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < kWorkspaceHeader || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    return apply::launch_cols(src, dst, layers, rows, cols * elem_bytes, static_cast<int64_t>(block_cols) * elem_bytes,
+                              elem_bytes, perm, perm_layer_stride, workspace, s);
 }
 
 int dtp_down_weight_workspace_size(int H_kv, int R, int d, int N, size_t* bytes) {

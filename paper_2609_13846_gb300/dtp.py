@@ -74,6 +74,11 @@ def lib():
     L.dtp_search_chain_ex.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp,
                                       _vp, _vp, _sz, _vp]
     L.dtp_chain_score.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+    L.dtp_head_writes_workspace_size.argtypes = [ctypes.POINTER(_sz)]
+    L.dtp_head_writes.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
+    L.dtp_layout_order.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
+    L.dtp_permute_rows.argtypes = [_vp, _vp, _i32, _i64, _i64, _i32, _vp, _i64, _vp, _sz, _vp]
+    L.dtp_permute_cols.argtypes = [_vp, _vp, _i32, _i64, _i64, _i32, _i32, _vp, _i64, _vp, _sz, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -81,6 +86,8 @@ def lib():
                                             _vp]
     for fn in ("dtp_search_chain_workspace_size", "dtp_search_chain", "dtp_search_chain_ex", "dtp_chain_score",
                "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
+               "dtp_head_writes_workspace_size", "dtp_head_writes", "dtp_layout_order", "dtp_permute_rows",
+               "dtp_permute_cols",
                "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
                "dtp_down_weight_workspace_size", "dtp_down_weight_sqnorm", "dtp_down_finalize",
@@ -487,3 +494,125 @@ def chain_score(S_up: torch.Tensor, S_down: torch.Tensor | None, h: torch.Tensor
     if check:
         _check("dtp_chain_score (device status)", workspace_status(workspace, stream))
     return out
+
+
+# ------------------------------------------------------------ producer / apply --
+
+def _status_workspace(dev, stream) -> torch.Tensor:
+    n = _sz(0)
+    _check("dtp_head_writes_workspace_size", lib().dtp_head_writes_workspace_size(ctypes.byref(n)))
+    return _keep(torch.empty(n.value, dtype=torch.uint8, device=dev), stream)
+
+
+def head_writes(attn: torch.Tensor, W_o: torch.Tensor, gamma: torch.Tensor, rms: torch.Tensor, head_dim: int,
+                q_per_row: int = 1, out: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                stream=None, check: bool = False) -> torch.Tensor:
+    """C[j,t,:] = gamma * (sum of a_{h,t} W_o^(h)T over the heads of row j) / rms[t] (Sec. 3), bf16.
+
+    attn [T, H_q*head_dim] and W_o [d, H_q*head_dim] bf16 CUDA; gamma [d] and
+    rms [T] fp32.  Returns C [H_q/q_per_row, T, d] bf16.
+    """
+    for name, t in (("attn", attn), ("W_o", W_o)):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    T, K = attn.shape
+    d = W_o.shape[0]
+    if W_o.shape != (d, K) or K % head_dim:
+        raise ValueError("W_o must be [d, H_q*head_dim] with attn [T, H_q*head_dim]")
+    Hq = K // head_dim
+    if q_per_row < 1 or Hq % q_per_row:
+        raise ValueError("q_per_row must divide H_q")
+    if gamma.shape != (d,) or gamma.dtype != torch.float32 or rms.shape != (T,) or rms.dtype != torch.float32:
+        raise ValueError("gamma must be fp32 [d] and rms fp32 [T]")
+    if out is None:
+        out = torch.empty((Hq // q_per_row, T, d), dtype=torch.bfloat16, device=attn.device)
+    if workspace is None:
+        workspace = _status_workspace(attn.device, stream)
+    st = lib().dtp_head_writes(_ptr(attn), _ptr(W_o), _ptr(gamma.contiguous()), _ptr(rms.contiguous()), T, d, Hq,
+                               head_dim, q_per_row, _ptr(out), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_head_writes", st)
+    if check:
+        _check("dtp_head_writes (device status)", workspace_status(workspace, stream))
+    return out
+
+
+def layout_order(labels: torch.Tensor, D: int, balanced: bool = True, stream=None, check: bool = True) -> torch.Tensor:
+    """order[i][p]: layer i's items listed device by device (each device's in increasing index).
+
+    labels [layers, n] (or [n]) int32 CUDA: head_part or neuron_dev.
+    """
+    lab = labels.unsqueeze(0) if labels.dim() == 1 else labels
+    if lab.dtype != torch.int32 or not lab.is_cuda or not lab.is_contiguous():
+        raise ValueError("labels must be a contiguous int32 CUDA tensor")
+    Lyr, n = lab.shape
+    order = torch.empty_like(lab)
+    ws = _status_workspace(lab.device, stream)
+    st = lib().dtp_layout_order(_ptr(lab), Lyr, n, D, int(balanced), _ptr(order), _ptr(ws), ws.numel(),
+                                _stream(stream))
+    _check("dtp_layout_order", st)
+    if check:
+        _check("dtp_layout_order (device status)", workspace_status(ws, stream))
+    return order if labels.dim() == 2 else order[0]
+
+
+def permute_rows(src: torch.Tensor, perm: torch.Tensor, block_rows: int = 1, out: torch.Tensor | None = None,
+                 stream=None, check: bool = True) -> torch.Tensor:
+    """dst[i][b*B + r] = src[i][perm[i][b]*B + r] for src [layers, rows, ...] (or [rows, ...]), perm [layers, rows/B]."""
+    x = src.unsqueeze(0) if perm.dim() == 1 else src
+    pm = perm.unsqueeze(0) if perm.dim() == 1 else perm
+    if not x.is_contiguous() or not pm.is_contiguous() or pm.dtype != torch.int32:
+        raise ValueError("src and perm must be contiguous, perm int32")
+    Lyr, rows = x.shape[0], x.shape[1]
+    row_bytes = x[0, 0].numel() * x.element_size()
+    dst = torch.empty_like(x) if out is None else (out.unsqueeze(0) if perm.dim() == 1 else out)
+    ws = _status_workspace(x.device, stream)
+    st = lib().dtp_permute_rows(_ptr(x), _ptr(dst), Lyr, rows, row_bytes, block_rows, _ptr(pm), pm.shape[1],
+                                _ptr(ws), ws.numel(), _stream(stream))
+    _check("dtp_permute_rows", st)
+    if check:
+        _check("dtp_permute_rows (device status)", workspace_status(ws, stream))
+    return dst[0] if perm.dim() == 1 else dst
+
+
+def permute_cols(src: torch.Tensor, perm: torch.Tensor, block_cols: int = 1, out: torch.Tensor | None = None,
+                 stream=None, check: bool = True) -> torch.Tensor:
+    """dst[i][r][b*B + c] = src[i][r][perm[i][b]*B + c] for src [layers, rows, cols] (or [rows, cols])."""
+    x = src.unsqueeze(0) if perm.dim() == 1 else src
+    pm = perm.unsqueeze(0) if perm.dim() == 1 else perm
+    if x.dim() != 3 or not x.is_contiguous() or not pm.is_contiguous() or pm.dtype != torch.int32:
+        raise ValueError("src must be contiguous [layers, rows, cols] and perm contiguous int32")
+    Lyr, rows, cols = x.shape
+    dst = torch.empty_like(x) if out is None else (out.unsqueeze(0) if perm.dim() == 1 else out)
+    ws = _status_workspace(x.device, stream)
+    st = lib().dtp_permute_cols(_ptr(x), _ptr(dst), Lyr, rows, cols, x.element_size(), block_cols, _ptr(pm),
+                                pm.shape[1], _ptr(ws), ws.numel(), _stream(stream))
+    _check("dtp_permute_cols", st)
+    if check:
+        _check("dtp_permute_cols (device status)", workspace_status(ws, stream))
+    return dst[0] if perm.dim() == 1 else dst
+
+
+def apply_layout(W: dict, h: torch.Tensor, nu: torch.Tensor, D: int, head_dim: int, stream=None,
+                 check: bool = True) -> tuple[dict, torch.Tensor, torch.Tensor]:
+    """Permute dense weights for a layout so that device l's KV groups and neurons are the l-th
+    contiguous shard (Sec. 3).
+
+    W holds q [.., Hq*hd, d], k and v [.., G*hd, d], o [.., d, Hq*hd], gate and
+    up [.., N, d], down [.., d, N], with an optional leading layers axis that
+    h [layers, G] and nu [layers, N] then share.  Other entries are copied by
+    reference.  Returns (permuted weights, head order, neuron order).
+    """
+    ho = layout_order(h, D, stream=stream, check=check)
+    no = layout_order(nu, D, stream=stream, check=check)
+    G = h.shape[-1]
+    hq = W["q"].shape[-2] // head_dim
+    blk = (hq // G) * head_dim
+    out = dict(W)
+    out["q"] = permute_rows(W["q"], ho, blk, stream=stream, check=check)
+    out["k"] = permute_rows(W["k"], ho, head_dim, stream=stream, check=check)
+    out["v"] = permute_rows(W["v"], ho, head_dim, stream=stream, check=check)
+    out["o"] = permute_cols(W["o"], ho, blk, stream=stream, check=check)
+    out["gate"] = permute_rows(W["gate"], no, 1, stream=stream, check=check)
+    out["up"] = permute_rows(W["up"], no, 1, stream=stream, check=check)
+    out["down"] = permute_cols(W["down"], no, 1, stream=stream, check=check)
+    return out, ho, no
