@@ -211,9 +211,11 @@ def layout_suite(args, w, S_up, S_down, S_add, stream):
     def run(check):
         out = {}
         for k, (mh, mn, mini) in dev_masks.items():
-            out[k] = dtp.search_chain(S_up, Sd, D, w.iters, workspace=ws, check=check, move_heads=mh,
-                                      move_neurons=mn, minimize=mini)
-            out[k] = {"J": out[k]["J"].clone(), "iters": out[k]["iters_done"].clone()}
+            r = dtp.search_chain(S_up, Sd, D, w.iters, workspace=ws, check=check, move_heads=mh,
+                                 move_neurons=mn, minimize=mini)
+            out[k] = {"J": r["J"].clone(), "iters": r["iters_done"].clone()}
+            if k == "optimised":
+                out[k].update(h=r["h"].clone(), nu=r["nu"].clone())
         if S_add is not None:
             r = dtp.search_chain(S_add, Sd, D, w.iters, workspace=ws, check=check)
             sc = dtp.chain_score(S_up, Sd, r["h"], r["nu"], D, workspace=ws, check=check)
@@ -236,7 +238,39 @@ def layout_suite(args, w, S_up, S_down, S_add, stream):
     return {"D": D, "ms": s0.elapsed_time(s1), "J": {k: v for k, v in J.items() if not k.startswith("random")},
             "J_random_mean": round(sum(rnd) / len(rnd), 4), "J_random_range": [min(rnd), max(rnd)],
             "J_random_expected": (2 * Lyr - 1) / D,
-            "layouts": len(res)}
+            "layouts": len(res)}, (res["optimised"]["h"], res["optimised"]["nu"], D)
+
+
+def time_apply(w, h, nu, D, stream):
+    """Apply the optimised layout to stacked synthetic weights of every layer (q/k/v/o, gate/up/down),
+    captured once in a CUDA graph and timed over graph replays (inputs resident, 3 replays)."""
+    from paper_2609_13846_gb300 import dtp
+    Wt = synth.make_dense_weights(w.layers, w.d, w.G * w.q_per_group, w.G, w.head_dim, w.N, seed=w.seed + 3000,
+                                  device=h.device)
+    fn = lambda: dtp.apply_layout(Wt, h, nu, D, w.head_dim, check=False)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        fn()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        out, ho, no = fn()
+    g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(3):
+        g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / 3
+    # the graph's result is the layout's: device l's groups and neurons are the l-th contiguous slice
+    ok = all(bool((h[i][ho[i]] == torch.arange(D, device=h.device).repeat_interleave(w.G // D)).all())
+             for i in range(w.layers))
+    nbytes = 2 * sum(v.numel() * v.element_size() for v in Wt.values())
+    return {"ms": ms, "bytes": nbytes, "GBs": nbytes / ms / 1e6, "launches": 9, "graph": True, "shards_ok": ok}
 
 
 def run_model(args):
@@ -257,9 +291,24 @@ def run_model(args):
     S_add = torch.zeros((Lyr, G, N), dtype=torch.float32, device=dev) if args.add_score else None
     t_aff = t_down = t_add = 0.0
     q = args.qheads
+    t_prod = 0.0
+    if args.producer and q not in (1, w.q_per_group):
+        raise SystemExit("--producer takes --qheads 1 (KV-group rows) or the model's query heads per group")
     for i in range(Lyr):
         L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
             synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
+        if args.producer:
+            # C from the attention outputs: one row per query head, or per KV group when q == 1
+            P = synth.make_attention_inputs(T, d, G * w.q_per_group, w.head_dim, w.layer_seed(i) + 2000, device=dev)
+            torch.cuda.synchronize()
+            p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            p0.record(stream)
+            L["C"] = dtp.head_writes(P["attn"], P["W_o"], P["gamma"], P["rms"], w.head_dim,
+                                     1 if q > 1 else w.q_per_group, out=L["C"])
+            p1.record(stream)
+            torch.cuda.synchronize()
+            t_prod += p0.elapsed_time(p1)
+            del P
         Dn = synth.make_down_inputs(d, G, w.qkv_rows, N, T, seed=w.seed + 1000 + i, device=dev)
         act2 = torch.zeros(N, dtype=torch.float32, device=dev)
         A = S_up[i]
@@ -306,18 +355,21 @@ def run_model(args):
         torch.cuda.synchronize()
         searches[f"D{D}"] = {"ms": s0.elapsed_time(s1) / 3, "J": float(r["J"]), "J_random": (2 * Lyr - 1) / D,
                              "iters_done": int(r["iters_done"])}
-    suite = layout_suite(args, w, S_up, S_down, S_add if args.add_score else None, stream)
-    total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values())
+    suite, (h_opt, nu_opt, D_opt) = layout_suite(args, w, S_up, S_down, S_add if args.add_score else None, stream)
+    apply = time_apply(w, h_opt, nu_opt, D_opt, stream)
+    total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values()) + t_prod + t_add
     chunk = (16 // q) * q                      # query heads per launch; each launch has its own X pass
     fl = 2.0 * d * 2 * N * (G * q + -(-(G * q) // chunk)) * T * Lyr
     line = {"metric": f"whole-model affinity + layout time ({args.model})", "value": total_ms / 1e3, "unit": "s",
             "higher_is_better": False, "n_gpus": 1, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": args.model, "layers": Lyr, "d": d, "G": G, "N": N, "T_per_layer": T,
-                       "query_heads_per_group": q,
+                       "query_heads_per_group": q, "producer": bool(args.producer),
                        "D": list(w.D), "iters": w.iters, "qkv_rows": w.qkv_rows},
             "affinity_ms": t_aff, "affinity_tflops": fl / (t_aff / 1e3) / 1e12,
             "layer_tokens_per_s": Lyr * T / (t_aff / 1e3), "down_edge_ms": t_down, "search": searches,
-            "add_affinity_ms": t_add if args.add_score else None, "layout_suite": suite,
+            "add_affinity_ms": t_add if args.add_score else None, "layout_suite": suite, "apply": apply,
+            "pipeline_s": (total_ms + suite["ms"] + apply["ms"]) / 1e3,
+            "producer_ms": t_prod if args.producer else None,
             "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s"}
     print(json.dumps(line), flush=True)
 
@@ -333,6 +385,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--model", default=None, help="time a whole-model pipeline instead, e.g. qwen3_0.6b_model")
     ap.add_argument("--add-score", action="store_true", help="with --model: also the ADD affinity and its layout")
+    ap.add_argument("--producer", action="store_true",
+                    help="with --model: make C from synthetic attention outputs with the producer kernel")
     ap.add_argument("--qheads", type=int, default=1,
                     help="with --model: query heads per KV group; >1 scores each query head and sums per group")
     args = ap.parse_args()

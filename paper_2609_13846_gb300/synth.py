@@ -49,6 +49,8 @@ class Workload:
     outliers: bool = True
     iters: int = 10
     qkv_rows: int = 512   # next layer's q/k/v rows per KV group: (query heads per group + 2) * head_dim
+    head_dim: int = 128
+    q_per_group: int = 2  # query heads per KV group
 
     def layer_seed(self, layer: int) -> int:
         """Seed of layer ``layer``: the workload seed plus the layer index."""
@@ -58,15 +60,16 @@ class Workload:
 # The five calibration workloads.  FLOP per token of the affinity pass is
 # 2*d*2N*(G+1).
 WORKLOADS = {
-    "tiny": Workload("tiny", d=64, G=2, N=128, T=256, D=(2,), dtype="f32", seed=0, outliers=False, qkv_rows=64),
+    "tiny": Workload("tiny", d=64, G=2, N=128, T=256, D=(2,), dtype="f32", seed=0, outliers=False, qkv_rows=64,
+                     head_dim=16),
     "qwen3_0.6b_layer": Workload("qwen3_0.6b_layer", d=1024, G=8, N=3072, T=16384, D=(2,),
                                  dtype="bf16", seed=1),
     "qwen3_0.6b_model": Workload("qwen3_0.6b_model", d=1024, G=8, N=3072, T=65536, D=(2, 4),
                                  dtype="bf16", layers=28, seed=100),
     "danube3_500m_model": Workload("danube3_500m_model", d=1536, G=8, N=4096, T=65536, D=(4,),
-                                   dtype="bf16", layers=16, seed=200, qkv_rows=384),
+                                   dtype="bf16", layers=16, seed=200, qkv_rows=384, head_dim=96),
     "llama3.1_8b_layer": Workload("llama3.1_8b_layer", d=4096, G=8, N=14336, T=32768, D=(4, 8),
-                                  dtype="bf16", seed=3, qkv_rows=768),
+                                  dtype="bf16", seed=3, qkv_rows=768, q_per_group=4),
 }
 
 
@@ -153,3 +156,32 @@ def make_down_inputs(d: int, G: int, R: int, N: int, T: int, seed: int, *, dtype
         out = {k: v.to(torch.bfloat16) for k, v in out.items()}
     out["rms"] = rms
     return out
+
+
+def make_attention_inputs(T: int, d: int, Hq: int, head_dim: int, seed: int, *, device="cpu"):
+    """Seeded stand-ins for the producer of C (Sec. 3: p_h = gamma . (a_h W_o^(h)T) / r).
+
+    attn [T, Hq*head_dim] bf16: the heads' outputs before o_proj, N(0,1) with
+    head h scaled by s_h log-uniform in [0.1, 1]; W_o [d, Hq*head_dim] bf16:
+    N(0, 0.02^2); gamma [d] fp32: 1 + N(0, 0.1^2); rms [T] fp32: uniform in
+    [0.5, 1.5].  Draw order as listed (the head scales first).
+    """
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed))
+    u = torch.rand((Hq,), generator=gen, device=device, dtype=torch.float32)
+    scales = torch.exp(math.log(0.1) * (1.0 - u)).repeat_interleave(head_dim)
+    attn = (_randn(gen, (T, Hq * head_dim), device) * scales).to(torch.bfloat16)
+    W_o = (_randn(gen, (d, Hq * head_dim), device) * 0.02).to(torch.bfloat16)
+    gamma = 1.0 + 0.1 * _randn(gen, (d,), device)
+    rms = 0.5 + torch.rand((T,), generator=gen, device=device, dtype=torch.float32)
+    return dict(attn=attn, W_o=W_o, gamma=gamma, rms=rms)
+
+
+def make_dense_weights(layers: int, d: int, Hq: int, G: int, head_dim: int, N: int, seed: int, *, device="cpu"):
+    """Stacked bf16 stand-ins for a model's permuted weights [layers, ...]: q [Hq*hd, d], k and v
+    [G*hd, d], o [d, Hq*hd], gate and up [N, d], down [d, N], all N(0, 0.02^2), drawn in that order."""
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed))
+    shapes = dict(q=(Hq * head_dim, d), k=(G * head_dim, d), v=(G * head_dim, d), o=(d, Hq * head_dim),
+                  gate=(N, d), up=(N, d), down=(d, N))
+    return {k: (_randn(gen, (layers, *sh), device) * 0.02).to(torch.bfloat16) for k, sh in shapes.items()}
