@@ -111,6 +111,30 @@ int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate,
                                void* stream);
 
 /*
+ * Launch options of the bf16 affinity pass.
+ *   max_ctas   0: one persistent CTA per SM (the default of the other entry
+ *              points); n > 0: at most n CTAs, leaving the other SMs to
+ *              kernels running concurrently on other streams (for instance the
+ *              layout search of the previous layer, which runs on one SM)
+ *   reserved   must be zero
+ */
+typedef struct dtp_affinity_opts {
+    int max_ctas;
+    int reserved[7];
+} dtp_affinity_opts;
+
+/*
+ * dtp_affinity_accumulate_ex with launch options (opts non-NULL).  The
+ * result does not depend on max_ctas (the reduction order is fixed by the
+ * work units, not by the grid).  The fp32 mode ignores the options.  Same
+ * workspace and errors as dtp_affinity_accumulate_ex.
+ */
+int dtp_affinity_accumulate_opts(const void* X, const void* C, const void* W_gate, const void* W_up,
+                                 const float* rms_next, int64_t T, int d, int H_kv, int N, int dtype,
+                                 float* A, float* act2, const dtp_affinity_opts* opts, void* workspace,
+                                 size_t workspace_bytes, void* stream);
+
+/*
  * The first-order score per query head, summed over the query heads of each
  * KV group (Sec. 3, "Affinity scores": E_t[Delta_hk^2] is taken per query head
  * h from that head's own write p_h, and the group's score is the sum of its

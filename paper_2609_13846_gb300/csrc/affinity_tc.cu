@@ -488,9 +488,11 @@ size_t workspace_bytes_with_act(int64_t T, int d, int G, int N) {
     return align_up(workspace_bytes(T, d, G, N), 256) + static_cast<size_t>(NT * TC) * BNEU * sizeof(float);
 }
 
-// G heads of C; A receives G / qpg rows (qpg consecutive heads summed per row).
+// G heads of C; A receives G / qpg rows (qpg consecutive heads summed per row).  max_ctas > 0
+// caps the persistent grid below one CTA per SM (leaving SMs to concurrent kernels).
 int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N,
-                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg) {
+                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg,
+                   int max_ctas) {
     if (qpg < 1 || G % qpg) return DTP_ERR_ARG;
     CUtensorMap m_wg, m_wu, m_x, m_c;
     const cuuint64_t row_stride = static_cast<cuuint64_t>(d) * 2;
@@ -523,7 +525,8 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev));
     DTP_CUDA_TRY(cudaFuncSetAttribute(affinity_fo_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       static_cast<int>(kSmemBytes)));
-    const int grid = static_cast<int>(p.units < sms ? p.units : sms);
+    const int cap = (max_ctas > 0 && max_ctas < sms) ? max_ctas : sms;
+    const int grid = static_cast<int>(p.units < cap ? p.units : cap);
     // chunk grouping: keep the weight tiles of the units in flight within a third of L2
     {
         const double tile_bytes = 2.0 * BNEU * d * 2.0;
@@ -550,7 +553,7 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
 
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
            void* workspace, cudaStream_t stream, const float* rms, float* act2) {
-    return launch_grouped(X, C, Wg, Wu, T, d, G, N, A, workspace, stream, rms, act2, 1);
+    return launch_grouped(X, C, Wg, Wu, T, d, G, N, A, workspace, stream, rms, act2, 1, 0);
 }
 
 }  // namespace tc

@@ -12,7 +12,8 @@ size_t workspace_bytes_with_act(int64_t T, int d, int G, int N);
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
            void* workspace, cudaStream_t stream, const float* rms, float* act2);
 int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N,
-                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg);
+                   float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg,
+                   int max_ctas);
 }  // namespace tc
 namespace f32 {
 size_t workspace_bytes(int64_t T, int d, int G, int N);
@@ -146,6 +147,31 @@ int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate,
                        static_cast<const float*>(W_up), T, d, H_kv, N, A, workspace, s, rms_next, act2);
 }
 
+int dtp_affinity_accumulate_opts(const void* X, const void* C, const void* W_gate, const void* W_up,
+                                 const float* rms_next, int64_t T, int d, int H_kv, int N, int dtype, float* A,
+                                 float* act2, const dtp_affinity_opts* opts, void* workspace, size_t workspace_bytes,
+                                 void* stream) {
+    if (!opts || opts->max_ctas < 0) return DTP_ERR_ARG;
+    for (int i = 0; i < 7; ++i)
+        if (opts->reserved[i] != 0) return DTP_ERR_ARG;
+    if (dtype != DTP_BF16 || opts->max_ctas == 0)
+        return dtp_affinity_accumulate_ex(X, C, W_gate, W_up, rms_next, T, d, H_kv, N, dtype, A, act2, workspace,
+                                          workspace_bytes, stream);
+    if (!affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
+    if ((rms_next == nullptr) != (act2 == nullptr)) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;
+    if (!X || !C || !W_gate || !W_up || !A) return DTP_ERR_ARG;
+    if (!aligned16(X) || !aligned16(C) || !aligned16(W_gate) || !aligned16(W_up) || !aligned16(A))
+        return DTP_ERR_ARG;
+    const bool with_act = act2 != nullptr;
+    if (with_act && (!aligned16(act2) || !aligned16(rms_next))) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < affinity_ws(T, d, H_kv, N, dtype, with_act) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    return tc::launch_grouped(X, C, W_gate, W_up, T, d, H_kv, N, A, workspace, s, rms_next, act2, 1, opts->max_ctas);
+}
+
 int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, const void* W_up, int64_t T, int d,
                             int H_kv, int N, int dtype, float* A, void* workspace, size_t workspace_bytes,
                             void* stream) {
@@ -186,7 +212,8 @@ int dtp_affinity_accumulate_grouped(const void* X, const void* C_q, const void* 
         const float* r = h0 == 0 ? rms_next : nullptr;   // the activation term once, with the first chunk
         float* a2 = h0 == 0 ? act2 : nullptr;
         const int st = dtype == DTP_BF16
-                           ? tc::launch_grouped(X, Cc, W_gate, W_up, T, d, hc, N, Ac, workspace, s, r, a2, q_per_group)
+                           ? tc::launch_grouped(X, Cc, W_gate, W_up, T, d, hc, N, Ac, workspace, s, r, a2, q_per_group,
+                                                0)
                            : f32::launch_grouped(static_cast<const float*>(X), static_cast<const float*>(Cc),
                                                  static_cast<const float*>(W_gate), static_cast<const float*>(W_up), T,
                                                  d, hc, N, Ac, workspace, s, r, a2, q_per_group);

@@ -32,6 +32,11 @@ _i32 = ctypes.c_int
 _sz = ctypes.c_size_t
 
 
+class AffinityOpts(ctypes.Structure):
+    """dtp_affinity_opts: max_ctas caps the persistent grid (0 = one CTA per SM)."""
+    _fields_ = [("max_ctas", ctypes.c_int), ("reserved", ctypes.c_int * 7)]
+
+
 class DTPError(RuntimeError):
     """A libdtp call returned a non-zero dtp_status."""
 
@@ -64,6 +69,8 @@ def lib():
     L.dtp_affinity_add_grouped_workspace_size.argtypes = [_i64, _i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_affinity_add_accumulate_grouped.argtypes = [_vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _sz,
                                                       _vp]
+    L.dtp_affinity_accumulate_opts.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp,
+                                               ctypes.POINTER(AffinityOpts), _vp, _sz, _vp]
     L.dtp_affinity_add_workspace_size.argtypes = [_i64, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_affinity_add_accumulate.argtypes = [_vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
     L.dtp_down_weight_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
@@ -87,6 +94,7 @@ def lib():
     for fn in ("dtp_search_chain_workspace_size", "dtp_search_chain", "dtp_search_chain_ex", "dtp_chain_score",
                "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
                "dtp_head_writes_workspace_size", "dtp_head_writes", "dtp_layout_order", "dtp_permute_rows",
+               "dtp_affinity_accumulate_opts",
                "dtp_permute_cols",
                "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
@@ -155,11 +163,12 @@ def affinity_workspace(T: int, d: int, H_kv: int, N: int, dtype: int, device) ->
 
 def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
                         A: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
-                        stream=None) -> torch.Tensor:
+                        stream=None, max_ctas: int = 0) -> torch.Tensor:
     """A[h,k] += sum_t Delta_{t,h,k}^2 (Sec. 3); returns A [H_kv, N] fp32 on X's device.
 
     X [T,d], C [H_kv,T,d], W_gate/W_up [N,d]: contiguous CUDA tensors, all bf16
     or all fp32.  ``A`` is accumulated into (a zero tensor is made if None).
+    max_ctas > 0 caps the bf16 kernel's persistent grid (SMs left to other streams).
     """
     for name, t in (("X", X), ("C", C), ("W_gate", W_gate), ("W_up", W_up)):
         if not t.is_cuda or not t.is_contiguous():
@@ -178,6 +187,13 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
         raise ValueError("A must be a contiguous fp32 [H_kv, N] tensor on X's device")
     if workspace is None:
         workspace = affinity_workspace(T, d, H, N, code, X.device)
+    if max_ctas:
+        opts = AffinityOpts(max_ctas=int(max_ctas))
+        st = lib().dtp_affinity_accumulate_opts(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), None, T, d, H, N, code,
+                                                _ptr(A), None, ctypes.byref(opts), _ptr(workspace), workspace.numel(),
+                                                _stream(stream))
+        _check("dtp_affinity_accumulate_opts", st)
+        return A
     st = lib().dtp_affinity_accumulate(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, code, _ptr(A),
                                        _ptr(workspace), workspace.numel(), _stream(stream))
     _check("dtp_affinity_accumulate", st)

@@ -6,6 +6,8 @@ times, with nothing else in between, so that an ncu capture with
 
     python -m paper_2609_13846_gb300.profile_case --what affinity --workload qwen3_0.6b_layer --launches 2
     python -m paper_2609_13846_gb300.profile_case --what search --workload qwen3_0.6b_model --D 4 --layers 28
+    python -m paper_2609_13846_gb300.profile_case --what producer --workload qwen3_0.6b_layer --qrow 1
+    python -m paper_2609_13846_gb300.profile_case --what gather --workload qwen3_0.6b_model --layers 28
 """
 from __future__ import annotations
 
@@ -18,7 +20,8 @@ from . import dtp, synth
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--what", choices=["affinity", "search"], default="affinity")
+    ap.add_argument("--what", choices=["affinity", "search", "producer", "gather"], default="affinity")
+    ap.add_argument("--qrow", type=int, default=1, help="producer: query heads per output row")
     ap.add_argument("--workload", default="qwen3_0.6b_layer")
     ap.add_argument("--T", type=int, default=None, help="token count (default: the workload's)")
     ap.add_argument("--launches", type=int, default=2)
@@ -37,6 +40,27 @@ def main():
             dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"], A=A, workspace=ws)
         torch.cuda.synchronize()
         print(f"affinity {args.workload} T={T}: {args.launches} launches, A sum {float(A.sum()):.6e}")
+    elif args.what == "producer":
+        T = args.T or w.T
+        P = synth.make_attention_inputs(T, w.d, w.G * w.q_per_group, w.head_dim, w.seed, device=dev)
+        C = torch.empty(((w.G * w.q_per_group) // args.qrow, T, w.d), dtype=torch.bfloat16, device=dev)
+        torch.cuda.synchronize()
+        for _ in range(args.launches):
+            dtp.head_writes(P["attn"], P["W_o"], P["gamma"], P["rms"], w.head_dim, args.qrow, out=C)
+        torch.cuda.synchronize()
+        print(f"producer {args.workload} T={T} rows={C.shape[0]}: {args.launches} launches")
+    elif args.what == "gather":
+        Wt = synth.make_dense_weights(args.layers, w.d, w.G * w.q_per_group, w.G, w.head_dim, w.N, w.seed,
+                                      device=dev)
+        D = args.D or w.D[-1]
+        nu = torch.stack([torch.randperm(w.N, device=dev) % D for _ in range(args.layers)]).to(torch.int32)
+        no = dtp.layout_order(nu, D)
+        torch.cuda.synchronize()
+        for _ in range(args.launches):
+            dtp.permute_cols(Wt["down"], no, 1, check=False)
+            dtp.permute_rows(Wt["gate"], no, 1, check=False)
+        torch.cuda.synchronize()
+        print(f"gather {args.workload} layers={args.layers}: {args.launches} launches each")
     else:
         As = torch.stack([synth.make_affinity_matrix(w.G, w.N, seed=w.seed + i, device="cpu")
                           for i in range(args.layers)]).to(dev).contiguous()

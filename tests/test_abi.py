@@ -135,3 +135,18 @@ def test_chain_score_and_ablation_reject_before_launch(lib):
                                    ctypes.c_size_t(1 << 16), None) == -1
     # too small a workspace
     assert lib.dtp_chain_score(p, p, 2, 8, 32, 4, p, p, None, p, p, p, ctypes.c_size_t(16), None) == -5
+
+
+def test_affinity_opts_reject_bad_options(lib):
+    from paper_2609_13846_gb300 import dtp
+    buf = ctypes.create_string_buffer(1 << 12)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    bad = dtp.AffinityOpts(max_ctas=-1)
+    assert lib.dtp_affinity_accumulate_opts(p, p, p, p, None, 16, 64, 2, 128, 0, p, None, ctypes.byref(bad), p,
+                                            ctypes.c_size_t(1 << 12), None) == -1
+    res = dtp.AffinityOpts(max_ctas=4)
+    res.reserved[3] = 1
+    assert lib.dtp_affinity_accumulate_opts(p, p, p, p, None, 16, 64, 2, 128, 0, p, None, ctypes.byref(res), p,
+                                            ctypes.c_size_t(1 << 12), None) == -1
+    assert lib.dtp_affinity_accumulate_opts(p, p, p, p, None, 16, 64, 2, 128, 0, p, None, None, p,
+                                            ctypes.c_size_t(1 << 12), None) == -1

@@ -153,3 +153,14 @@ def test_full_size_sampled_neurons(name):
     got = A[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
     assert _rel_fro(got, ref) <= BF16_TOL
     assert torch.isfinite(A).all() and (A >= 0).all()
+
+
+@pytest.mark.parametrize("max_ctas", [1, 7, 151])
+def test_grid_cap_does_not_change_the_result(max_ctas):
+    """The persistent grid may be capped (SMs left to a concurrent search); A is bitwise the same."""
+    L = synth.make_layer(1024, 8, 3072, 2048, seed=12, dtype="bf16")
+    g = {k: v.to(DEV) for k, v in L.items()}
+    full = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"])
+    capped = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"], max_ctas=max_ctas)
+    torch.cuda.synchronize()
+    assert torch.equal(full, capped)
