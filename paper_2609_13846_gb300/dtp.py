@@ -414,7 +414,9 @@ def search_layout_batched(A: torch.Tensor, D: int, iters: int, workspace: torch.
                score=torch.empty(Lyr, dtype=torch.float64, device=dev),
                iters_done=torch.empty(Lyr, dtype=torch.int32, device=dev))
     if workspace is None:
-        workspace = torch.empty(search_workspace_size(Lyr, H, N, D), dtype=torch.uint8, device=dev)
+        workspace = _keep(torch.empty(search_workspace_size(Lyr, H, N, D), dtype=torch.uint8, device=dev), stream)
+    for t in out.values():
+        _keep(t, stream)
     st = lib().dtp_search_layout_batched(_ptr(A), Lyr, H, N, D, iters, _ptr(out["h"]), _ptr(out["nu"]),
                                          _ptr(out["score_q"]), _ptr(out["score"]), _ptr(out["iters_done"]),
                                          _ptr(workspace), workspace.numel(), _stream(stream))
@@ -471,6 +473,8 @@ def search_chain(S_up: torch.Tensor, S_down: torch.Tensor | None, D: int, iters:
                J_q=torch.empty((), dtype=torch.int64, device=dev),
                J=torch.empty((), dtype=torch.float64, device=dev),
                iters_done=torch.empty((), dtype=torch.int32, device=dev))
+    for t in out.values():
+        _keep(t, stream)
     mh = _device_mask(move_heads, Lyr, dev, stream)
     mn = _device_mask(move_neurons, Lyr, dev, stream)
     if workspace is None:
