@@ -144,7 +144,11 @@ def test_full_size_sampled_neurons(name):
     w = synth.WORKLOADS[name]
     L = synth.make_workload_layer(w, device=DEV)
     A = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"])
+    # the benchmark's step caps the grid at one CTA below the SM count (the search runs beside it)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    A_capped = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"], max_ctas=sms - 1)
     torch.cuda.synchronize()
+    assert torch.equal(A, A_capped)
     rng = np.random.default_rng(0)
     cols = np.sort(rng.choice(w.N, size=6, replace=False))
     cols = np.unique(np.concatenate([cols, [0, w.N - 1]]))
