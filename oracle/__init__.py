@@ -70,6 +70,9 @@ def _load():
     lib.oracle_search_layout.argtypes = [_f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                          _i32p, _i32p, _i64p, _f64p, _i32p, _i32p]
     lib.oracle_search_layout.restype = ctypes.c_int
+    lib.oracle_global_layout.argtypes = [_f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p, _i64p,
+                                         _f64p, _i32p]
+    lib.oracle_global_layout.restype = ctypes.c_int
     lib.oracle_head_writes.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
                                        ctypes.c_int, ctypes.c_int, _f64p]
     lib.oracle_head_writes.restype = None
@@ -256,6 +259,24 @@ def search_layout(A, D: int, iters: int):
         raise ValueError(f"oracle_search_layout: status {st}")
     return dict(h=h, nu=nu, score_q=int(sq.value), score=float(sc.value), iters_done=int(it.value),
                 unique=bool(uq.value))
+
+
+def global_layout(A, D: int):
+    """The exact maximum of one layer's up-edge J over every balanced layout (Sec. 3 'Objective'):
+    the best exact neuron step over the unlabelled head partitions, each in its canonical labelling,
+    the first (lexicographic) best one kept.  dict(h, nu, score_q, score, parts)."""
+    A = _c(A, np.float32)
+    G, N = A.shape
+    h = np.zeros(G, dtype=np.int32)
+    nu = np.zeros(N, dtype=np.int32)
+    sq = ctypes.c_int64(0)
+    sc = ctypes.c_double(0.0)
+    npart = ctypes.c_int(0)
+    st = _load().oracle_global_layout(_p(A, _f32p), G, N, D, _p(h, _i32p), _p(nu, _i32p), ctypes.byref(sq),
+                                      ctypes.byref(sc), ctypes.byref(npart))
+    if st != 0:
+        raise ValueError(f"oracle_global_layout: status {st}")
+    return dict(h=h, nu=nu, score_q=sq.value, score=sc.value, parts=npart.value)
 
 
 def hungarian_max(W):

@@ -31,6 +31,8 @@
  *   oracle_normalize_unit_mass, oracle_chain_search
  *                          Sec. 3 "Objective" (Eq. objective, both sums) and
  *                          "Optimiser" over all layers of a model.
+ *   oracle_global_layout   Sec. 3 "Objective": the exact maximum of one layer's
+ *                          up-edge J over all layouts (unlabelled partitions).
  *   oracle_head_writes     Sec. 3 "Affinity scores": head h's write into the
  *                          FFN input, p_h = gamma . (a_h W_o^(h)) / r.
  *   oracle_layout_order    Sec. 3 (sharding a permuted dense model): the
@@ -786,6 +788,84 @@ int oracle_chain_edge_scores(const float* S_up, const float* S_down, int L, int 
     }
     free(n);
     return bad;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Global optimum of one layer's up-edge objective                           */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * J(h, nu) of one layer is unchanged when the device labels of h and nu are
+ * permuted together, so its maximum is the best exact neuron step over the
+ * UNLABELLED balanced head partitions: G!/((G/D)!^D D!) of them (35 for G=8,
+ * D=2; 105 for D=4).  Each is visited once through its canonical labelling
+ * (a restricted growth string: a device label first appears after all
+ * smaller ones), generated recursively in lexicographic order; the first
+ * partition with the largest exact neuron-step value wins, with that step's
+ * lexicographically smallest nu.  This is the stronger reference the ascent
+ * is measured against.
+ */
+typedef struct {
+    const int64_t* q;
+    int G, N, D, cap;
+    int* cur;        /* [G] labels being built */
+    int* cnt;        /* [D] heads per device so far */
+    int64_t* M;      /* [N][D] */
+    int* nu_tmp;     /* [N] */
+    int64_t best;
+    int* h_best;
+    int* nu_best;
+    int parts;
+    int status;
+} global_ctx;
+
+static void global_rec(global_ctx* c, int k, int used) {
+    if (c->status != OR_OK) return;
+    if (k == c->G) {
+        build_gain(c->q, c->G, c->N, c->D, c->cur, c->M);
+        int uniq = 1;
+        int st = neuron_step_from_gain(c->M, c->N, c->D, c->nu_tmp, &uniq, 0);
+        if (st != OR_OK) { c->status = st; return; }
+        int64_t v = 0;
+        for (int i = 0; i < c->N; ++i) v += c->M[(int64_t)i * c->D + c->nu_tmp[i]];
+        ++c->parts;
+        if (v > c->best) {
+            c->best = v;
+            memcpy(c->h_best, c->cur, sizeof(int) * (size_t)c->G);
+            memcpy(c->nu_best, c->nu_tmp, sizeof(int) * (size_t)c->N);
+        }
+        return;
+    }
+    /* label l: an existing device with room, or the next unused one */
+    for (int l = 0; l <= used && l < c->D; ++l) {
+        if (c->cnt[l] == c->cap) continue;
+        c->cur[k] = l;
+        ++c->cnt[l];
+        global_rec(c, k + 1, l == used ? used + 1 : used);
+        --c->cnt[l];
+    }
+}
+
+int oracle_global_layout(const float* A, int G, int N, int D, int* h, int* nu, int64_t* score_q, double* score,
+                         int* n_parts) {
+    if (D < 2 || D > OR_DMAX || G <= 0 || G % D || G > OR_GMAX || N <= 0 || N % D) return OR_ERR_ARG;
+    int64_t* q = (int64_t*)malloc(sizeof(int64_t) * (size_t)G * N);
+    int status = oracle_quantize(A, G, N, q, NULL);
+    if (status != OR_OK) { free(q); return status; }
+    int cur[OR_GMAX], cnt[OR_DMAX];
+    memset(cnt, 0, sizeof(cnt));
+    global_ctx c = {q, G, N, D, G / D, cur, cnt, (int64_t*)malloc(sizeof(int64_t) * (size_t)N * D),
+                    (int*)malloc(sizeof(int) * (size_t)N), -1, h, nu, 0, OR_OK};
+    global_rec(&c, 0, 0);
+    int64_t total = 0;
+    for (int64_t i = 0; i < (int64_t)G * N; ++i) total += q[i];
+    if (c.status == OR_OK) {
+        *score_q = c.best;
+        *score = total > 0 ? (double)c.best / (double)total : 0.0;
+        *n_parts = c.parts;
+    }
+    free(c.M); free(c.nu_tmp); free(q);
+    return c.status;
 }
 
 /* ------------------------------------------------------------------------ */

@@ -269,3 +269,69 @@ def test_search_d8_single_partition_is_global():
                for nu in [oracle.neuron_step(q, np.arange(8, dtype=np.int32), 8)[0]])
     assert res["score_q"] == best
     assert res["iters_done"] == 2
+
+
+# ------------------------------------------------- global optimum (Sec. 3 "Objective") ----
+
+import itertools as _it  # noqa: E402
+import math as _math  # noqa: E402
+
+
+def _balanced_labelings(n, D):
+    cap = n // D
+    for a in _it.product(range(D), repeat=n):
+        if all(a.count(l) == cap for l in range(D)):
+            yield np.array(a, dtype=np.int32)
+
+
+@pytest.mark.parametrize("G,N,D,seed", [(4, 8, 2, 0), (4, 8, 2, 1), (6, 6, 3, 2), (4, 8, 4, 3), (2, 10, 2, 4)])
+def test_global_layout_against_brute_force(G, N, D, seed):
+    """The maximum over every labelled head partition and every balanced assignment equals the
+    best exact neuron step over the unlabelled partitions; the ascent never exceeds it."""
+    A = synth.make_affinity_matrix(G, N, seed=seed).numpy()
+    q, _ = oracle.quantize(A)
+    best = max(oracle.layout_score(q, h, nu) for h in _balanced_labelings(G, D) for nu in _balanced_labelings(N, D))
+    g = oracle.global_layout(A, D)
+    assert g["score_q"] == best == oracle.layout_score(q, g["h"], g["nu"])
+    assert oracle.search_layout(A, D, 10)["score_q"] <= best
+
+
+@pytest.mark.parametrize("G,D", [(8, 2), (8, 4), (8, 8), (6, 3), (6, 2), (4, 2), (12, 3), (12, 4), (16, 2)])
+def test_global_layout_visits_every_unlabelled_partition_once(G, D):
+    A = synth.make_affinity_matrix(G, 2 * D, seed=G + D).numpy()
+    g = oracle.global_layout(A, D)
+    cap = G // D
+    assert g["parts"] == _math.factorial(G) // (_math.factorial(cap) ** D * _math.factorial(D))
+    # canonical labelling: balanced, and each label first appears after every smaller one
+    h = g["h"].tolist()
+    assert all(h.count(l) == cap for l in range(D))
+    firsts = [h.index(l) for l in range(D)]
+    assert firsts == sorted(firsts) and firsts[0] == 0
+
+
+def test_global_layout_ties_take_the_first_canonical_partition():
+    """Tie-heavy integer affinities: the winner is the first canonical partition (in lexicographic
+    order) reaching the maximum, with its lexicographically smallest optimal assignment."""
+    G, N, D = 4, 8, 2
+    for seed in range(6):
+        A = synth.make_affinity_matrix(G, N, seed=50 + seed, kind="integer").numpy()
+        q, _ = oracle.quantize(A)
+        canon = [h for h in _balanced_labelings(G, D) if list(h).index(1) > 0 and h[0] == 0]
+        best, first = -1, None
+        for h in sorted(canon, key=tuple):
+            nu, _ = oracle.neuron_step(q, h, D)
+            v = oracle.layout_score(q, h, nu)
+            if v > best:
+                best, first = v, (h, nu)
+        g = oracle.global_layout(A, D)
+        assert g["score_q"] == best
+        np.testing.assert_array_equal(g["h"], first[0])
+        np.testing.assert_array_equal(g["nu"], first[1])
+
+
+def test_global_layout_with_one_head_per_device_is_one_neuron_step():
+    A = synth.make_affinity_matrix(8, 64, seed=9).numpy()
+    g = oracle.global_layout(A, 8)
+    assert g["parts"] == 1
+    one = oracle.search_layout(A, 8, 1)
+    assert g["score_q"] == one["score_q"]
