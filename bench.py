@@ -514,6 +514,17 @@ def main():
         model_search[f"D{Dm}_ms"] = m0.elapsed_time(m1) / 5
         model_search[f"D{Dm}_mean_score"] = float(rm["score"].mean())
         model_search[f"D{Dm}_max_iters_done"] = int(rm["iters_done"].max())
+        # the exact optimum of every layer (all unlabelled head partitions), beside the ascent
+        rg = dtp.search_global(A_model, Dm)
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        rg = dtp.search_global(A_model, Dm, check=False)
+        g1.record(stream)
+        torch.cuda.synchronize()
+        model_search[f"D{Dm}_global_ms"] = g0.elapsed_time(g1)
+        model_search[f"D{Dm}_global_mean_score"] = float(rg["score"].mean())
+        model_search[f"D{Dm}_ascent_over_global_min"] = float((rm["score_q"].double() / rg["score_q"].double()).min())
+        model_search[f"D{Dm}_layers_at_global"] = int((rm["score_q"] == rg["score_q"]).sum())
     del A_model
 
     # ---- end to end through the public API, host buffers in pinned memory.  Every step copies its

@@ -361,6 +361,31 @@ int dtp_search_chain(const float* S_up, const float* S_down, int layers, int H_k
                      int32_t* iters_done, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * The exact maximum of each layer's up-edge objective over every balanced
+ * layout (Sec. 3 "Objective": J of one layer, Sec. 3 "Optimiser" uses it only
+ * through the ascent; this is the reference the ascent is measured against).
+ * J is unchanged when device labels are permuted jointly in h and nu, so the
+ * maximum is the best exact neuron step over the unlabelled balanced head
+ * partitions, H_kv! / ((H_kv/D)!^D D!) of them (35 for H_kv=8, D=2; 105 for
+ * D=4; 1 for D=8).  Each partition is taken in its canonical labelling (a
+ * device label first appears after every smaller one); the first partition in
+ * lexicographic order with the largest value wins, with its exact neuron
+ * step's lexicographically smallest assignment.  Arithmetic and A as in
+ * dtp_search_layout_batched (score_q exact, score = score_q / sum q).
+ *   A           [layers, H_kv, N] fp32, device
+ *   head_part   [layers, H_kv] int32 out (canonical labels)
+ *   neuron_dev  [layers, N] int32 out;  score_q [layers] int64, score [layers]
+ *               double out
+ * Size rules of dtp_search_layout, and at most 2^20 unlabelled partitions per
+ * layer.  Workspace from dtp_search_global_workspace_size.  Asynchronous;
+ * invalid entries are reported through the workspace status word.
+ */
+int dtp_search_global_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes);
+int dtp_search_global(const float* A, int layers, int H_kv, int N, int D, int32_t* head_part,
+                      int32_t* neuron_dev, int64_t* score_q, double* score, void* workspace,
+                      size_t workspace_bytes, void* stream);
+
+/*
  * dtp_search_chain with the ablations of Sec. 3 ("Optimiser"; the layouts of
  * Table 4): restricting which layers move, freezing heads or neurons, or
  * minimising J (the anti-optimised layout).

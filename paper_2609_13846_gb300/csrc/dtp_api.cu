@@ -54,6 +54,10 @@ int64_t partition_count(int G, int D);
 int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* head, int32_t* nu, int64_t* score_q,
            double* score, int32_t* iters_done, void* workspace, cudaStream_t stream);
 size_t chain_workspace_bytes(int Lyr, int G, int N, int D);
+int64_t unlabelled_count(int G, int D);
+size_t global_workspace_bytes(int layers, int G, int N, int D);
+int launch_global(const float* A, int layers, int G, int N, int D, int32_t* head, int32_t* nu, int64_t* score_q,
+                  double* score, void* workspace, cudaStream_t stream);
 int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, int iters,
                  const uint8_t* move_heads, const uint8_t* move_neurons, int minimize, int32_t* head, int32_t* nu,
                  int64_t* J_q, double* J, int32_t* iters_done, void* workspace, cudaStream_t stream);
@@ -392,6 +396,29 @@ int dtp_search_layout_batched(const float* A, int layers, int H_kv, int N, int D
     if (!workspace || workspace_bytes < need || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
     return search::launch(A, layers, H_kv, N, D, iters, head_part, neuron_dev, score_q, score, iters_done, workspace,
                           static_cast<cudaStream_t>(stream));
+}
+
+// The exhaustive search visits at most 2^20 unlabelled partitions per layer.
+static bool global_sizes_ok(int layers, int H, int N, int D) {
+    return search_sizes_ok(layers, H, N, D, 1) && layers <= 65535 &&
+           search::unlabelled_count(H, D) <= (int64_t(1) << 20) &&
+           static_cast<int64_t>(layers) * search::unlabelled_count(H, D) <= (int64_t(1) << 26);
+}
+
+int dtp_search_global_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes) {
+    if (!bytes || !global_sizes_ok(layers, H_kv, N, D)) return DTP_ERR_ARG;
+    *bytes = search::global_workspace_bytes(layers, H_kv, N, D);
+    return DTP_OK;
+}
+
+int dtp_search_global(const float* A, int layers, int H_kv, int N, int D, int32_t* head_part, int32_t* neuron_dev,
+                      int64_t* score_q, double* score, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!global_sizes_ok(layers, H_kv, N, D)) return DTP_ERR_ARG;
+    if (!A || !head_part || !neuron_dev || !score_q || !score || !aligned16(A)) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < search::global_workspace_bytes(layers, H_kv, N, D) || !aligned16(workspace))
+        return DTP_ERR_WORKSPACE;
+    return search::launch_global(A, layers, H_kv, N, D, head_part, neuron_dev, score_q, score, workspace,
+                                 static_cast<cudaStream_t>(stream));
 }
 
 int dtp_search_chain_workspace_size(int layers, int H_kv, int N, int D, size_t* bytes) {

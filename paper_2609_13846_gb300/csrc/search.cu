@@ -677,6 +677,239 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     }
 }
 
+// ------------------------------------------------ global optimum (one layer) --
+//
+// J of one layer is unchanged when the device labels of h and nu are permuted
+// together, so its maximum is the best exact neuron step over the UNLABELLED
+// balanced head partitions, G!/((G/D)!^D D!) of them.  Each is taken in its
+// canonical labelling (a label first appears after every smaller one), in
+// lexicographic order; one block runs the exact neuron step of one (layer,
+// partition) item, and a second kernel takes, per layer, the first partition
+// with the largest value and recomputes its assignment.
+
+__host__ __device__ inline uint64_t fact_u64(int n) {
+    uint64_t f = 1;
+    for (int i = 2; i <= n; ++i) f *= static_cast<uint64_t>(i);
+    return f;
+}
+
+// Completions of a canonical prefix: r heads left, `used` labelled blocks with
+// rem[] places left, D - used blocks not yet opened (cap places each, opened
+// in order): r! / (prod rem! * cap!^(D-used) * (D-used)!).  r <= 16.
+__device__ uint64_t rgs_completions(int r, const int* rem, int used, int D, int cap) {
+    uint64_t n = fact_u64(r);
+    for (int l = 0; l < used; ++l) n /= fact_u64(rem[l]);
+    const int u = D - used;
+    const uint64_t fc = fact_u64(cap);
+    for (int i = 0; i < u; ++i) n /= fc;
+    return n / fact_u64(u);
+}
+
+// The idx-th canonical balanced labelling in lexicographic order (thread-local).
+__device__ bool unrank_canonical(uint64_t idx, int G, int D, int* h) {
+    const int cap = G / D;
+    int cnt[DMAX];
+    for (int l = 0; l < DMAX; ++l) cnt[l] = 0;
+    int used = 0;
+    for (int k = 0; k < G; ++k) {
+        bool placed = false;
+        for (int l = 0; l <= used && l < D; ++l) {
+            if (cnt[l] == cap) continue;
+            ++cnt[l];
+            const int used2 = l == used ? used + 1 : used;
+            int rem[DMAX];
+            for (int a = 0; a < used2; ++a) rem[a] = cap - cnt[a];
+            const uint64_t c = rgs_completions(G - k - 1, rem, used2, D, cap);
+            if (idx < c) {
+                h[k] = l;
+                used = used2;
+                placed = true;
+                break;
+            }
+            idx -= c;
+            --cnt[l];
+        }
+        if (!placed) return false;
+    }
+    return true;
+}
+
+int64_t unlabelled_count(int G, int D) {
+    const int cap = G / D;
+    uint64_t n = fact_u64(G);
+    for (int l = 0; l < D; ++l) n /= fact_u64(cap);
+    return static_cast<int64_t>(n / fact_u64(D));
+}
+
+// Validity, the fixed-point exponent and the total of q of the layer in L.A.
+__device__ bool layer_prologue(Layer& L, Shared& sh, int64_t* total_out) {
+    const int64_t GN = static_cast<int64_t>(L.G) * L.N;
+    uint32_t amax_bits = 0;
+    int bad = 0;
+    for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
+        const float a = L.A[i];
+        if (!(a >= 0.0f) || isinf(a)) bad = 1;
+        else amax_bits = max(amax_bits, __float_as_uint(a));
+    }
+    bad = __syncthreads_or(bad);
+    const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
+    if (bad) return false;
+    const float amax = __uint_as_float(static_cast<uint32_t>(amax_all));
+    int e = 0;
+    if (amax > 0.0f) frexpf(amax, &e);
+    L.e = e;
+    if (total_out) {
+        int64_t part = 0;
+        for (int64_t i = threadIdx.x; i < GN; i += kThreads) part += quantize(L.A[i], e);
+        *total_out = block_sum_i64(part, sh);
+    }
+    return true;
+}
+
+// Layer view over the block's buffer (and an smem copy of A in mode 2).
+__device__ void layer_view(Layer& L, const float* A_glob, int G, int N, int D, uint8_t* buf, int use_smem) {
+    L.A = A_glob;
+    L.G = G;
+    L.N = N;
+    L.D = D;
+    L.cap = N / D;
+    L.M = reinterpret_cast<int64_t*>(buf);
+    L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * D * sizeof(int64_t));
+    if (use_smem == 2) {
+        float* As = reinterpret_cast<float*>(buf + align_up_dev(static_cast<size_t>(N) * D * sizeof(int64_t) +
+                                                                static_cast<size_t>(N) * sizeof(int32_t), 16));
+        for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) As[i] = A_glob[i];
+        __syncthreads();
+        L.A = As;
+    }
+}
+
+template <int DT>
+__device__ int64_t assignment_value(const Layer& L, Shared& sh) {
+    int64_t part = 0;
+    for (int k = threadIdx.x; k < L.N; k += kThreads) part += L.M[static_cast<int64_t>(k) * DT + L.nu[k]];
+    return block_sum_i64(part, sh);
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads, 1)
+global_items_kernel(const float* __restrict__ A_all, int layers, int G, int N, int64_t n_unl,
+                    int64_t* __restrict__ values, int* __restrict__ ws_status, uint8_t* __restrict__ gbuf,
+                    size_t per_block, int use_smem) {
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ Shared sh;
+    uint8_t* buf = use_smem ? dsm : gbuf + static_cast<size_t>(blockIdx.x) * per_block;
+    const int64_t items = static_cast<int64_t>(layers) * n_unl;
+    for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+        const int layer = static_cast<int>(item / n_unl);
+        const int64_t pidx = item - static_cast<int64_t>(layer) * n_unl;
+        Layer L;
+        layer_view(L, A_all + static_cast<int64_t>(layer) * G * N, G, N, DT, buf, use_smem);
+        if (threadIdx.x == 0) {
+            sh.status = DTP_OK;
+            for (int l = 0; l < DMAX; ++l) sh.pi[l] = 0;
+            int hh[GMAX];
+            if (!unrank_canonical(static_cast<uint64_t>(pidx), G, DT, hh)) sh.status = DTP_ERR_NOT_CONVERGED;
+            for (int g = 0; g < G; ++g) sh.h[g] = hh[g];
+        }
+        if (!layer_prologue(L, sh, nullptr)) {
+            if (threadIdx.x == 0) {
+                values[item] = -1;
+                atomicMin(ws_status, static_cast<int>(DTP_ERR_ARG));
+            }
+            __syncthreads();
+            continue;
+        }
+        build_gain<DT>(L, sh);
+        if constexpr (DT == 2) neuron_step_d2(L, sh);
+        else neuron_step_general<DT>(L, sh);
+        __syncthreads();
+        if (sh.status != DTP_OK) {
+            if (threadIdx.x == 0) {
+                values[item] = -1;
+                atomicMin(ws_status, sh.status);
+            }
+            __syncthreads();
+            continue;
+        }
+        const int64_t v = assignment_value<DT>(L, sh);
+        if (threadIdx.x == 0) values[item] = v;
+        __syncthreads();
+    }
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads, 1)
+global_pick_kernel(const float* __restrict__ A_all, int G, int N, int64_t n_unl, const int64_t* __restrict__ values,
+                   int32_t* __restrict__ head_out, int32_t* __restrict__ nu_out, int64_t* __restrict__ score_q_out,
+                   double* __restrict__ score_out, int* __restrict__ ws_status, uint8_t* __restrict__ gbuf,
+                   size_t per_block, int use_smem) {
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ Shared sh;
+    const int layer = blockIdx.x;
+    const int64_t* vals = values + static_cast<int64_t>(layer) * n_unl;
+    // first index of the largest value (values < 0 mark failed items)
+    int64_t best = -1;
+    int best_idx = 0x7FFFFFFF;
+    for (int64_t i = threadIdx.x; i < n_unl; i += kThreads) better(best, best_idx, vals[i], static_cast<int>(i));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const int64_t s2 = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+        const int i2 = __shfl_xor_sync(0xFFFFFFFFu, best_idx, o);
+        better(best, best_idx, s2, i2);
+    }
+    if (lane == 0) sh.red_i64[warp] = best, sh.red_int[warp] = best_idx;
+    __syncthreads();
+    if (warp == 0) {
+        int64_t b = sh.red_i64[lane];
+        int bi = sh.red_int[lane];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const int64_t s2 = __shfl_xor_sync(0xFFFFFFFFu, b, o);
+            const int i2 = __shfl_xor_sync(0xFFFFFFFFu, bi, o);
+            better(b, bi, s2, i2);
+        }
+        if (lane == 0) {
+            sh.J = b;
+            sh.best_idx = bi;
+        }
+    }
+    __syncthreads();
+    if (sh.J < 0) {                                   // every item failed: already reported
+        if (threadIdx.x == 0) atomicMin(ws_status, static_cast<int>(DTP_ERR_ARG));
+        return;
+    }
+    uint8_t* buf = use_smem ? dsm : gbuf + static_cast<size_t>(blockIdx.x) * per_block;
+    Layer L;
+    layer_view(L, A_all + static_cast<int64_t>(layer) * G * N, G, N, DT, buf, use_smem);
+    if (threadIdx.x == 0) {
+        sh.status = DTP_OK;
+        for (int l = 0; l < DMAX; ++l) sh.pi[l] = 0;
+        int hh[GMAX];
+        unrank_canonical(static_cast<uint64_t>(sh.best_idx), G, DT, hh);
+        for (int g = 0; g < G; ++g) sh.h[g] = hh[g];
+    }
+    int64_t total = 0;
+    layer_prologue(L, sh, &total);
+    build_gain<DT>(L, sh);
+    if constexpr (DT == 2) neuron_step_d2(L, sh);
+    else neuron_step_general<DT>(L, sh);
+    __syncthreads();
+    if (sh.status != DTP_OK) {
+        if (threadIdx.x == 0) atomicMin(ws_status, sh.status);
+        return;
+    }
+    const int64_t v = assignment_value<DT>(L, sh);
+    for (int k = threadIdx.x; k < N; k += kThreads) nu_out[static_cast<int64_t>(layer) * N + k] = L.nu[k];
+    if (threadIdx.x < G) head_out[static_cast<int64_t>(layer) * G + threadIdx.x] = sh.h[threadIdx.x];
+    if (threadIdx.x == 0) {
+        score_q_out[layer] = v;
+        score_out[layer] = total > 0 ? static_cast<double>(v) / static_cast<double>(total) : 0.0;
+        if (v != sh.J) atomicMin(ws_status, static_cast<int>(DTP_ERR_NOT_CONVERGED));   // must recompute equal
+    }
+}
+
 // ------------------------------------------------------- whole-model search --
 //
 // Eq. objective with both sums: J = sum_i up_i + sum_{i<L-1} down_i, each matrix
@@ -1114,6 +1347,75 @@ int launch_chain(const float* S_up, const float* S_down, int Lyr, int G, int N, 
         default: return DTP_ERR_ARG;
     }
 #undef DTP_CHAIN_CASE
+}
+
+static size_t global_layout_bytes(int layers, int G, int N, int D, int grid, size_t* off_vals, size_t* off_gbuf) {
+    size_t o = kWorkspaceHeader;
+    *off_vals = o;
+    o += align_up(static_cast<size_t>(layers) * unlabelled_count(G, D) * sizeof(int64_t), 256);
+    *off_gbuf = o;
+    if (!fits_smem(N, D)) o += static_cast<size_t>(grid > layers ? grid : layers) * per_layer_bytes(N, D);
+    return o;
+}
+
+// The item kernel's grid: one block per SM, at most kGlobalMaxGrid (the workspace holds a
+// per-block buffer for that many blocks when the layer does not fit in shared memory).
+constexpr int kGlobalMaxGrid = 160;
+
+static int global_grid(int layers, int G, int D) {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev))
+        return -1;
+    if (sms > kGlobalMaxGrid) sms = kGlobalMaxGrid;
+    const int64_t items = static_cast<int64_t>(layers) * unlabelled_count(G, D);
+    return static_cast<int>(items < sms ? items : sms);
+}
+
+size_t global_workspace_bytes(int layers, int G, int N, int D) {
+    size_t a, b;
+    return global_layout_bytes(layers, G, N, D, kGlobalMaxGrid, &a, &b);
+}
+
+template <int DT>
+static int launch_global_t(const float* A, int layers, int G, int N, int32_t* head, int32_t* nu, int64_t* score_q,
+                           double* score, uint8_t* ws, cudaStream_t stream) {
+    const int grid = global_grid(layers, G, DT);
+    if (grid <= 0) return DTP_ERR_CUDA;
+    size_t o_vals, o_gbuf;
+    global_layout_bytes(layers, G, N, DT, grid, &o_vals, &o_gbuf);
+    int* ws_status = reinterpret_cast<int*>(ws);
+    int64_t* vals = reinterpret_cast<int64_t*>(ws + o_vals);
+    uint8_t* gbuf = ws + o_gbuf;
+    const bool smem = fits_smem(N, DT);
+    const int mode = !smem ? 0 : (with_a_bytes(G, N, DT) <= kSmemBudget ? 2 : 1);
+    const size_t dyn = mode == 2 ? with_a_bytes(G, N, DT) : (mode == 1 ? per_layer_bytes(N, DT) : 0);
+    const int64_t n_unl = unlabelled_count(G, DT);
+    DTP_CUDA_TRY(cudaFuncSetAttribute(global_items_kernel<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kSmemBudget)));
+    DTP_CUDA_TRY(cudaFuncSetAttribute(global_pick_kernel<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kSmemBudget)));
+    DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
+    global_items_kernel<DT><<<grid, kThreads, dyn, stream>>>(A, layers, G, N, n_unl, vals, ws_status, gbuf,
+                                                             per_layer_bytes(N, DT), mode);
+    global_pick_kernel<DT><<<layers, kThreads, dyn, stream>>>(A, G, N, n_unl, vals, head, nu, score_q, score,
+                                                              ws_status, gbuf, per_layer_bytes(N, DT), mode);
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
+}
+
+int launch_global(const float* A, int layers, int G, int N, int D, int32_t* head, int32_t* nu, int64_t* score_q,
+                  double* score, void* workspace, cudaStream_t stream) {
+    uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+    switch (D) {
+        case 2: return launch_global_t<2>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        case 3: return launch_global_t<3>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        case 4: return launch_global_t<4>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        case 5: return launch_global_t<5>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        case 6: return launch_global_t<6>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        case 7: return launch_global_t<7>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        case 8: return launch_global_t<8>(A, layers, G, N, head, nu, score_q, score, ws, stream);
+        default: return DTP_ERR_ARG;
+    }
 }
 
 int launch_chain_score(const float* S_up, const float* S_down, int Lyr, int G, int N, int D, const int32_t* head,

@@ -86,6 +86,8 @@ def lib():
     L.dtp_layout_order.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
     L.dtp_permute_rows.argtypes = [_vp, _vp, _i32, _i64, _i64, _i32, _vp, _i64, _vp, _sz, _vp]
     L.dtp_permute_cols.argtypes = [_vp, _vp, _i32, _i64, _i64, _i32, _i32, _vp, _i64, _vp, _sz, _vp]
+    L.dtp_search_global_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
+    L.dtp_search_global.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -94,7 +96,7 @@ def lib():
     for fn in ("dtp_search_chain_workspace_size", "dtp_search_chain", "dtp_search_chain_ex", "dtp_chain_score",
                "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
                "dtp_head_writes_workspace_size", "dtp_head_writes", "dtp_layout_order", "dtp_permute_rows",
-               "dtp_affinity_accumulate_opts",
+               "dtp_affinity_accumulate_opts", "dtp_search_global_workspace_size", "dtp_search_global",
                "dtp_permute_cols",
                "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
@@ -431,6 +433,34 @@ def search_layout(A: torch.Tensor, D: int, iters: int, workspace: torch.Tensor |
     """Coordinate ascent on one layer's A [H_kv, N]; tensors as in search_layout_batched, unbatched."""
     r = search_layout_batched(A.unsqueeze(0) if A.dim() == 2 else A, D, iters, workspace, stream, check)
     return {k: v[0] for k, v in r.items()}
+
+
+def search_global(A: torch.Tensor, D: int, workspace: torch.Tensor | None = None, stream=None,
+                  check: bool = True) -> dict:
+    """The exact maximum of each layer's up-edge J over every balanced layout (best exact neuron
+    step over the unlabelled head partitions).  A [L, H_kv, N] (or [H_kv, N]) fp32 CUDA.  Returns
+    h (canonical labels), nu, score_q, score; unbatched input gives unbatched outputs."""
+    x = A.unsqueeze(0) if A.dim() == 2 else A
+    if x.dtype != torch.float32 or not x.is_cuda or not x.is_contiguous():
+        raise ValueError("A must be a contiguous fp32 CUDA tensor [L, H_kv, N]")
+    Lyr, H, N = x.shape
+    dev = x.device
+    out = dict(h=torch.empty((Lyr, H), dtype=torch.int32, device=dev),
+               nu=torch.empty((Lyr, N), dtype=torch.int32, device=dev),
+               score_q=torch.empty(Lyr, dtype=torch.int64, device=dev),
+               score=torch.empty(Lyr, dtype=torch.float64, device=dev))
+    for t in out.values():
+        _keep(t, stream)
+    if workspace is None:
+        n = _sz(0)
+        _check("dtp_search_global_workspace_size", lib().dtp_search_global_workspace_size(Lyr, H, N, D, ctypes.byref(n)))
+        workspace = _keep(torch.empty(n.value, dtype=torch.uint8, device=dev), stream)
+    st = lib().dtp_search_global(_ptr(x), Lyr, H, N, D, _ptr(out["h"]), _ptr(out["nu"]), _ptr(out["score_q"]),
+                                 _ptr(out["score"]), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("dtp_search_global", st)
+    if check:
+        _check("dtp_search_global (device status)", workspace_status(workspace, stream))
+    return out if A.dim() == 3 else {k: v[0] for k, v in out.items()}
 
 
 def _chain_inputs(S_up: torch.Tensor, S_down: torch.Tensor | None):

@@ -150,3 +150,12 @@ def test_affinity_opts_reject_bad_options(lib):
                                             ctypes.c_size_t(1 << 12), None) == -1
     assert lib.dtp_affinity_accumulate_opts(p, p, p, p, None, 16, 64, 2, 128, 0, p, None, None, p,
                                             ctypes.c_size_t(1 << 12), None) == -1
+
+
+def test_global_search_size_rules(lib):
+    n = ctypes.c_size_t(0)
+    assert lib.dtp_search_global_workspace_size(28, 8, 3072, 4, ctypes.byref(n)) == 0
+    assert n.value >= 256 + 28 * 105 * 8
+    assert lib.dtp_search_global_workspace_size(1, 16, 64, 2, ctypes.byref(n)) == 0      # 6435 partitions
+    assert lib.dtp_search_global_workspace_size(1, 16, 64, 4, ctypes.byref(n)) == -1     # 2.6M partitions
+    assert lib.dtp_search_global_workspace_size(1, 8, 30, 4, ctypes.byref(n)) == -1      # D does not divide N

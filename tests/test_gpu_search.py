@@ -97,3 +97,40 @@ def test_search_is_deterministic():
     b = dtp.search_layout(A, 4, 10)
     for k in a:
         assert torch.equal(a[k], b[k])
+
+
+# ------------------------------------------------- global optimum of one layer ----
+
+@pytest.mark.parametrize("G,N,D,layers,kind", [
+    (8, 256, 2, 3, "lognormal"), (8, 3072, 4, 2, "lognormal"), (8, 3072, 2, 28, "lognormal"),
+    (6, 96, 3, 2, "lognormal"), (8, 64, 8, 2, "lognormal"), (4, 16, 2, 4, "integer"), (8, 128, 4, 3, "integer"),
+    (12, 48, 3, 1, "lognormal"), (16, 64, 2, 1, "lognormal")])
+def test_global_layout_matches_oracle(G, N, D, layers, kind):
+    As = np.stack([synth.make_affinity_matrix(G, N, seed=7 * i + N + D, kind=kind).numpy() for i in range(layers)])
+    r = dtp.search_global(torch.as_tensor(As, device=DEV).contiguous(), D)
+    asc = dtp.search_layout_batched(torch.as_tensor(As, device=DEV).contiguous(), D, 10)
+    for i in range(layers):
+        ref = oracle.global_layout(As[i], D)
+        np.testing.assert_array_equal(r["h"][i].cpu().numpy(), ref["h"])
+        np.testing.assert_array_equal(r["nu"][i].cpu().numpy(), ref["nu"])
+        assert int(r["score_q"][i]) == ref["score_q"]
+        assert float(r["score"][i]) == ref["score"]
+        assert int(asc["score_q"][i]) <= ref["score_q"]
+
+
+def test_global_layout_llama_width():
+    """N = 14336 (Llama-3.1-8B): M and nu do not fit in shared memory; per-block global buffers."""
+    A = synth.make_affinity_matrix(8, 14336, seed=3).numpy()
+    r = dtp.search_global(torch.as_tensor(A, device=DEV), 4)
+    ref = oracle.global_layout(A, 4)
+    np.testing.assert_array_equal(r["h"].cpu().numpy(), ref["h"])
+    np.testing.assert_array_equal(r["nu"].cpu().numpy(), ref["nu"])
+    assert int(r["score_q"]) == ref["score_q"]
+
+
+def test_global_layout_rejects_invalid_entries():
+    A = synth.make_affinity_matrix(8, 64, seed=1).numpy()
+    A[3, 5] = float("nan")
+    with pytest.raises(dtp.DTPError) as e:
+        dtp.search_global(torch.as_tensor(A, device=DEV), 2)
+    assert e.value.status == dtp.DTP_ERR_ARG
