@@ -149,6 +149,30 @@ __global__ void gather_cols_kernel(const uint8_t* __restrict__ src, uint8_t* __r
         } else if constexpr (MODE == kPack) {
             constexpr int kPer = static_cast<int>(16 / sizeof(E));
             const uint32_t be = static_cast<uint32_t>(block_elems);
+            // one column per block and 16-byte aligned permutation rows: the kPer entries behind
+            // an output word are read as whole 16-byte words (4 entries each)
+            const bool vec_perm = kPer % 4 == 0 && block_elems == 1 &&
+                                  (reinterpret_cast<uintptr_t>(pl) & 15) == 0;
+            if (vec_perm) {
+                for (int64_t o = lane; o < row_bytes / 16; o += 32) {
+                    union { uint4 v; E e[kPer]; } w;
+                    const int4* pv = reinterpret_cast<const int4*>(pl + o * kPer);
+#pragma unroll
+                    for (int q = 0; q < kPer / 4; ++q) {
+                        const int4 p4 = pv[q];
+                        const int32_t pe[4] = {p4.x, p4.y, p4.z, p4.w};
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const int64_t pb = pe[t];
+                            if (pb < 0 || pb >= nblocks) { bad = 1; w.e[4 * q + t] = E(0); continue; }
+                            w.e[4 * q + t] = reinterpret_cast<const E*>(s)[pb];
+                        }
+                    }
+                    *reinterpret_cast<uint4*>(d + o * 16) = w.v;
+                }
+                if (bad) atomicMin(status, static_cast<int>(DTP_ERR_ARG));
+                continue;
+            }
             for (int64_t o = lane; o < row_bytes / 16; o += 32) {
                 union { uint4 v; E e[kPer]; } w;
 #pragma unroll

@@ -169,3 +169,14 @@ def test_gathers_match_indexing(dtype, rows, cols, block):
         ri = np.concatenate([np.arange(b * rb, (b + 1) * rb) for b in pr[i]])
         assert torch.equal(got_c[i], src[i][:, ci])
         assert torch.equal(got_r[i], src[i][ri])
+
+
+def test_staged_column_gather_rejects_out_of_range_entries():
+    """One-column blocks of a bf16 matrix (the packed path with vector permutation reads); a bad entry is reported."""
+    src = torch.randn(4, 32, device=DEV).to(torch.bfloat16)
+    perm = torch.arange(32, dtype=torch.int32, device=DEV)
+    assert torch.equal(dtp.permute_cols(src, perm, 1), src)
+    perm[5] = 32
+    with pytest.raises(dtp.DTPError) as e:
+        dtp.permute_cols(src, perm, 1)
+    assert e.value.status == dtp.DTP_ERR_ARG
