@@ -8,6 +8,7 @@ times, with nothing else in between, so that an ncu capture with
     python -m paper_2609_13846_gb300.profile_case --what search --workload qwen3_0.6b_model --D 4 --layers 28
     python -m paper_2609_13846_gb300.profile_case --what producer --workload qwen3_0.6b_layer --qrow 1
     python -m paper_2609_13846_gb300.profile_case --what gather --workload qwen3_0.6b_model --layers 28
+    python -m paper_2609_13846_gb300.profile_case --what add --workload qwen3_0.6b_layer
 """
 from __future__ import annotations
 
@@ -20,7 +21,7 @@ from . import dtp, synth
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--what", choices=["affinity", "search", "producer", "gather"], default="affinity")
+    ap.add_argument("--what", choices=["affinity", "search", "producer", "gather", "add"], default="affinity")
     ap.add_argument("--qrow", type=int, default=1, help="producer: query heads per output row")
     ap.add_argument("--workload", default="qwen3_0.6b_layer")
     ap.add_argument("--T", type=int, default=None, help="token count (default: the workload's)")
@@ -40,6 +41,15 @@ def main():
             dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"], A=A, workspace=ws)
         torch.cuda.synchronize()
         print(f"affinity {args.workload} T={T}: {args.launches} launches, A sum {float(A.sum()):.6e}")
+    elif args.what == "add":
+        L = synth.make_workload_layer(w, T=args.T, device=dev)
+        T = L["X"].shape[0]
+        A = torch.zeros((w.G, w.N), dtype=torch.float32, device=dev)
+        torch.cuda.synchronize()
+        for _ in range(args.launches):
+            dtp.affinity_add_accumulate(L["C"], L["W_gate"], L["W_up"], A_add=A)
+        torch.cuda.synchronize()
+        print(f"add {args.workload} T={T}: {args.launches} launches, A sum {float(A.sum()):.6e}")
     elif args.what == "producer":
         T = args.T or w.T
         P = synth.make_attention_inputs(T, w.d, w.G * w.q_per_group, w.head_dim, w.seed, device=dev)
