@@ -277,24 +277,31 @@ def run_model(args):
     """Whole-model pipeline timing: every layer's affinity pass with the down-edge term on all
     its tokens, the ||w^d||^2 finalize, ||b_gk||^2 and S_down, then the whole-model search per D.
     Inputs are drawn per layer on the device outside the timed intervals."""
-    from paper_2609_13846_gb300 import dtp
+    from paper_2609_13846_gb300 import dtp, shard
     w = synth.WORKLOADS[args.model]
-    dev = torch.device("cuda", 0)
+    world, rank, local = dist_env()
+    dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
     stream = torch.cuda.current_stream()
     Lyr, G, N, T, d = w.layers, w.G, w.N, w.T, w.d
-    S_up = torch.empty((Lyr, G, N), dtype=torch.float32, device=dev)
-    S_down = torch.empty((max(Lyr - 1, 1), G, N), dtype=torch.float32, device=dev)
+    # under torchrun each rank scores its own block of layers (up edge and the down edge leaving
+    # each), then one all-gather hands every rank the whole model's matrices
+    mine = shard.layers_for_rank(Lyr, rank, world)
+    S_up_loc = torch.zeros((len(mine), G, N), dtype=torch.float32, device=dev)
+    S_down_loc = torch.zeros((len(mine), G, N), dtype=torch.float32, device=dev)
     ws = dtp.affinity_workspace(T, d, G, N, dtp.DTP_BF16, dev) if args.qheads == 1 else \
         torch.empty(dtp.affinity_grouped_workspace_size(T, d, G * args.qheads, args.qheads, N, dtp.DTP_BF16),
                     dtype=torch.uint8, device=dev)
-    S_add = torch.zeros((Lyr, G, N), dtype=torch.float32, device=dev) if args.add_score else None
+    S_add_loc = torch.zeros((len(mine), G, N), dtype=torch.float32, device=dev) if args.add_score else None
     t_aff = t_down = t_add = 0.0
     q = args.qheads
     t_prod = 0.0
     if args.producer and q not in (1, w.q_per_group):
         raise SystemExit("--producer takes --qheads 1 (KV-group rows) or the model's query heads per group")
-    for i in range(Lyr):
+    for li, i in enumerate(mine):
         L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
             synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
         if args.producer:
@@ -311,7 +318,7 @@ def run_model(args):
             del P
         Dn = synth.make_down_inputs(d, G, w.qkv_rows, N, T, seed=w.seed + 1000 + i, device=dev)
         act2 = torch.zeros(N, dtype=torch.float32, device=dev)
-        A = S_up[i]
+        A = S_up_loc[li]
         A.zero_()
         torch.cuda.synchronize()
         e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
@@ -326,14 +333,14 @@ def run_model(args):
         e1.record(stream)
         if i + 1 < Lyr:
             bn = dtp.down_weight_sqnorm(Dn["Wqkv"], Dn["gamma"], Dn["W_down"])
-            S_down[i].copy_(dtp.down_finalize(act2, bn, T))
+            S_down_loc[li].copy_(dtp.down_finalize(act2, bn, T))
         e2.record(stream)
         if args.add_score:
             e3 = torch.cuda.Event(enable_timing=True)
             if q == 1:
-                dtp.affinity_add_accumulate(L["C"], L["W_gate"], L["W_up"], A_add=S_add[i])
+                dtp.affinity_add_accumulate(L["C"], L["W_gate"], L["W_up"], A_add=S_add_loc[li])
             else:
-                dtp.affinity_add_accumulate_grouped(L["C"], L["W_gate"], L["W_up"], q, A_add=S_add[i])
+                dtp.affinity_add_accumulate_grouped(L["C"], L["W_gate"], L["W_up"], q, A_add=S_add_loc[li])
             e3.record(stream)
         torch.cuda.synchronize()
         t_aff += e0.elapsed_time(e1)
@@ -343,6 +350,20 @@ def run_model(args):
         del L, Dn
     if dtp.workspace_status(ws) != dtp.DTP_OK:
         raise RuntimeError("affinity kernel reported a device-side error")
+    torch.cuda.synchronize()
+    g0 = time.perf_counter()
+    S_up, S_down = shard.gather_model_affinities(S_up_loc, S_down_loc, Lyr, device=dev)
+    S_add = shard.gather_layer_results({"a": S_add_loc}, Lyr, device=dev)["a"] if args.add_score else None
+    torch.cuda.synchronize()
+    t_gather = (time.perf_counter() - g0) * 1e3 if world > 1 else 0.0
+    t_aff, t_down, t_add, t_prod = (shard.max_over_ranks(x, device=dev) for x in (t_aff, t_down, t_add, t_prod))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    if rank != 0:
+        return
+    if Lyr == 1:
+        S_down = S_up[:0]
     searches = {}
     for D in w.D:
         r = dtp.search_chain(S_up, S_down if Lyr > 1 else None, D, w.iters)
@@ -357,11 +378,12 @@ def run_model(args):
                              "iters_done": int(r["iters_done"])}
     suite, (h_opt, nu_opt, D_opt) = layout_suite(args, w, S_up, S_down, S_add if args.add_score else None, stream)
     apply = time_apply(w, h_opt, nu_opt, D_opt, stream)
-    total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values()) + t_prod + t_add
+    total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values()) + t_prod + t_add + t_gather
     chunk = (16 // q) * q                      # query heads per launch; each launch has its own X pass
     fl = 2.0 * d * 2 * N * (G * q + -(-(G * q) // chunk)) * T * Lyr
     line = {"metric": f"whole-model affinity + layout time ({args.model})", "value": total_ms / 1e3, "unit": "s",
-            "higher_is_better": False, "n_gpus": 1, "dtype": "bf16", "data": "synthetic",
+            "higher_is_better": False, "n_gpus": world, "scaling": "strong", "dtype": "bf16", "data": "synthetic",
+            "gather_ms": t_gather,
             "config": {"workload": args.model, "layers": Lyr, "d": d, "G": G, "N": N, "T_per_layer": T,
                        "query_heads_per_group": q, "producer": bool(args.producer),
                        "D": list(w.D), "iters": w.iters, "qkv_rows": w.qkv_rows},

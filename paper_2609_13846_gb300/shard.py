@@ -4,6 +4,12 @@ The up-edge objective (Sec. 3, Eq. objective, first sum) decouples across
 layers, and a layer's affinity depends only on that layer's calibration
 inputs, so a model's layers are split across ranks (one process per GPU) with
 no exchange on the data path.  Results are gathered once at the end.
+
+The whole-model objective (both sums) couples neighbouring layers, but its
+inputs do not: each rank scores the up edge of its layers and the down edge
+leaving each of them (which needs only the next layer's weights and the rms of
+its input), then one all-gather gives every rank the full set of matrices and
+the optimiser runs on them (milliseconds on one GPU).
 """
 from __future__ import annotations
 
@@ -53,3 +59,16 @@ def gather_layer_results(local: dict, n_layers: int, device=None) -> dict:
         dist.all_gather(parts, pad)
         out[name] = torch.cat([parts[r][: counts[r]] for r in range(world)], dim=0)
     return out
+
+
+def gather_model_affinities(S_up_local: torch.Tensor, S_down_local: torch.Tensor, n_layers: int,
+                            device=None) -> tuple[torch.Tensor, torch.Tensor]:
+    """All-gather a layer-sharded model's affinity matrices for the whole-model search.
+
+    S_up_local [n_mine, G, N]: the up edges of this rank's layers
+    (``layers_for_rank``); S_down_local [n_mine, G, N]: the down edge leaving
+    each of them (any values for the model's last layer, which has none).
+    Returns S_up [n_layers, G, N] and S_down [n_layers - 1, G, N] on every rank.
+    """
+    full = gather_layer_results({"up": S_up_local, "down": S_down_local}, n_layers, device=device)
+    return full["up"], full["down"][: max(n_layers - 1, 0)]
