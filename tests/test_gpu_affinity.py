@@ -168,3 +168,24 @@ def test_grid_cap_does_not_change_the_result(max_ctas):
     capped = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"], max_ctas=max_ctas)
     torch.cuda.synchronize()
     assert torch.equal(full, capped)
+
+
+@pytest.mark.parametrize("name", ["qwen3_0.6b_model", "danube3_500m_model"])
+def test_full_model_layer_sampled_neurons_with_down_term(name):
+    """Layer 0 of the full-model workloads (T = 65536 tokens) through the call the whole-model
+    benchmark makes (affinity pass with the down-edge activation term); the oracle computes
+    sampled neuron columns of A and entries of act2 over all tokens."""
+    w = synth.WORKLOADS[name]
+    L = synth.make_workload_layer(w, 0, device=DEV)
+    Dn = synth.make_down_inputs(w.d, w.G, w.qkv_rows, w.N, w.T, seed=w.seed + 1000, device=DEV)
+    A, act2 = dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"])
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(1)
+    cols = np.unique(np.concatenate([rng.choice(w.N, size=3, replace=False), [0, w.N - 1]]))
+    Lh = {k: v.cpu() for k, v in L.items()}
+    ref = _oracle(Lh, rows=cols)
+    got = A[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
+    assert _rel_fro(got, ref) <= BF16_TOL
+    ref_act = oracle.down_activation(Lh["X"].double().numpy(), Lh["W_gate"][cols].double().numpy(),
+                                     Lh["W_up"][cols].double().numpy(), Dn["rms"].double().cpu().numpy())
+    assert _rel_fro(act2[torch.as_tensor(cols, device=DEV)].double().cpu().numpy(), ref_act) <= BF16_TOL
