@@ -213,7 +213,18 @@ struct Layer {
     int G, N, D, cap, e;
     int64_t* M;   // [N][D]
     int32_t* nu;  // [N]
+    uint64_t* keys = nullptr;   // [N] selection keys, when M lives in global memory (else null)
 };
+
+// Bytes of M [N][D] int64 and nu [N] int32 (256-aligned); a layer kept in global memory also
+// has N uint64 selection keys after them.
+__host__ __device__ inline size_t mnu_bytes(int N, int D) {
+    const size_t b = static_cast<size_t>(N) * D * sizeof(int64_t) + static_cast<size_t>(N) * sizeof(int32_t);
+    return (b + 255) / 256 * 256;
+}
+__host__ __device__ inline size_t global_layer_bytes(int N, int D) {
+    return mnu_bytes(N, D) + (static_cast<size_t>(N) * sizeof(uint64_t) + 255) / 256 * 256;
+}
 
 template <int DT>
 __device__ void build_gain(const Layer& L, Shared& sh) {
@@ -354,7 +365,17 @@ __device__ void neuron_step_general(const Layer& L, Shared& sh) {
                 const int64_t v = mk[l] - alt;
                 return static_cast<uint64_t>(v) ^ (1ull << 63);
             };
-            const uint64_t t = block_select_desc(N, cap + 1, key, sh);
+            uint64_t t;
+            if (L.keys) {
+                // M is in global memory: form every key once, then the selection's passes read one
+                // word per neuron instead of D
+                for (int k = threadIdx.x; k < N; k += kThreads) L.keys[k] = key(k);
+                __syncthreads();
+                const uint64_t* ks = L.keys;
+                t = block_select_desc(N, cap + 1, [ks](int k) -> uint64_t { return ks[k]; }, sh);
+            } else {
+                t = block_select_desc(N, cap + 1, key, sh);
+            }
             if (threadIdx.x == 0) sh.pi[l] = static_cast<int64_t>(t ^ (1ull << 63));
             __syncthreads();
         }
@@ -604,6 +625,7 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     L.cap = N / D;
     L.M = reinterpret_cast<int64_t*>(buf);
     L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * D * sizeof(int64_t));
+    if (!use_smem) L.keys = reinterpret_cast<uint64_t*>(buf + mnu_bytes(N, D));
     if (use_smem == 2) {
         // A fits beside M and nu: copy it once; every pass then reads shared memory
         float* As = reinterpret_cast<float*>(buf + align_up_dev(static_cast<size_t>(N) * D * sizeof(int64_t) +
@@ -775,6 +797,7 @@ __device__ void layer_view(Layer& L, const float* A_glob, int G, int N, int D, u
     L.cap = N / D;
     L.M = reinterpret_cast<int64_t*>(buf);
     L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * D * sizeof(int64_t));
+    L.keys = use_smem ? nullptr : reinterpret_cast<uint64_t*>(buf + mnu_bytes(N, D));
     if (use_smem == 2) {
         float* As = reinterpret_cast<float*>(buf + align_up_dev(static_cast<size_t>(N) * D * sizeof(int64_t) +
                                                                 static_cast<size_t>(N) * sizeof(int32_t), 16));
@@ -1076,6 +1099,7 @@ chain_neuron_kernel(int Lyr, int G, int N, const int64_t* __restrict__ nbuf, con
     L.e = 0;
     L.M = reinterpret_cast<int64_t*>(buf);
     L.nu = reinterpret_cast<int32_t*>(buf + static_cast<size_t>(N) * DT * sizeof(int64_t));
+    if (!use_smem) L.keys = reinterpret_cast<uint64_t*>(buf + mnu_bytes(N, DT));
     const bool has_down = i + 1 < Lyr;
     if (threadIdx.x < G) {
         sh.h[threadIdx.x] = head[i * G + threadIdx.x];
@@ -1236,7 +1260,7 @@ static size_t with_a_bytes(int G, int N, int D) {
 size_t workspace_bytes(int layers, int G, int N, int D) {
     (void)G;
     size_t b = kWorkspaceHeader + align_up(static_cast<size_t>(layers) * sizeof(int), 256);
-    if (!fits_smem(N, D)) b += static_cast<size_t>(layers) * per_layer_bytes(N, D);
+    if (!fits_smem(N, D)) b += static_cast<size_t>(layers) * global_layer_bytes(N, D);
     return b;
 }
 
@@ -1260,7 +1284,7 @@ int launch(const float* A, int layers, int G, int N, int D, int iters, int32_t* 
     DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
     kern<<<layers, kThreads, dyn, stream>>>(A, G, N, D, iters, partition_count(G, D), head, nu, score_q,
                                                       score, iters_done, status, ws_status, gbuf,
-                                                      per_layer_bytes(N, D), mode);
+                                                      global_layer_bytes(N, D), mode);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
 }
@@ -1284,7 +1308,7 @@ static size_t chain_layout(int Lyr, int G, int N, int D, size_t* off_state, size
     *off_nbuf = o;
     o += align_up(static_cast<size_t>(2 * Lyr - 1) * GN * sizeof(int64_t), 256);
     *off_gbuf = o;
-    if (!fits_smem(N, D)) o += static_cast<size_t>(Lyr) * per_layer_bytes(N, D);
+    if (!fits_smem(N, D)) o += static_cast<size_t>(Lyr) * global_layer_bytes(N, D);
     return o;
 }
 
@@ -1318,7 +1342,7 @@ static int launch_chain_t(const float* S_up, const float* S_down, int Lyr, int G
     const uint32_t n_parts = static_cast<uint32_t>(partition_count(G, DT));
     for (int it = 0; it < iters; ++it) {
         chain_neuron_kernel<DT><<<Lyr, kThreads, dyn, stream>>>(Lyr, G, N, nbuf, head, nu, prices, st, ws_status, gbuf,
-                                                                 per_layer_bytes(N, DT), smem ? 1 : 0, move_neurons,
+                                                                 global_layer_bytes(N, DT), smem ? 1 : 0, move_neurons,
                                                                  minimize);
         chain_head_kernel<DT><<<Lyr, kThreads, 0, stream>>>(Lyr, G, N, nbuf, nu, head, layer_score, st, n_parts,
                                                              move_heads, minimize);
@@ -1354,7 +1378,7 @@ static size_t global_layout_bytes(int layers, int G, int N, int D, int grid, siz
     *off_vals = o;
     o += align_up(static_cast<size_t>(layers) * unlabelled_count(G, D) * sizeof(int64_t), 256);
     *off_gbuf = o;
-    if (!fits_smem(N, D)) o += static_cast<size_t>(grid > layers ? grid : layers) * per_layer_bytes(N, D);
+    if (!fits_smem(N, D)) o += static_cast<size_t>(grid > layers ? grid : layers) * global_layer_bytes(N, D);
     return o;
 }
 
@@ -1396,9 +1420,9 @@ static int launch_global_t(const float* A, int layers, int G, int N, int32_t* he
                                       static_cast<int>(kSmemBudget)));
     DTP_CUDA_TRY(cudaMemsetAsync(ws_status, 0, kWorkspaceHeader, stream));
     global_items_kernel<DT><<<grid, kThreads, dyn, stream>>>(A, layers, G, N, n_unl, vals, ws_status, gbuf,
-                                                             per_layer_bytes(N, DT), mode);
+                                                             global_layer_bytes(N, DT), mode);
     global_pick_kernel<DT><<<layers, kThreads, dyn, stream>>>(A, G, N, n_unl, vals, head, nu, score_q, score,
-                                                              ws_status, gbuf, per_layer_bytes(N, DT), mode);
+                                                              ws_status, gbuf, global_layer_bytes(N, DT), mode);
     DTP_CUDA_TRY(cudaGetLastError());
     return DTP_OK;
 }
