@@ -37,7 +37,7 @@ typedef enum {
     DTP_ERR_ARG = -1,            /* invalid size, pointer, alignment or combination      */
     DTP_ERR_CUDA = -2,           /* a CUDA runtime/driver call failed                      */
     DTP_ERR_NOT_CONVERGED = -3,  /* a bounded device loop or wait hit its limit            */
-    DTP_ERR_UNSUPPORTED = -4,    /* valid request this build does not handle (e.g. no GPU) */
+    DTP_ERR_UNSUPPORTED = -4,    /* valid request the library does not handle (e.g. no GPU) */
     DTP_ERR_WORKSPACE = -5       /* workspace NULL or smaller than the size query's value  */
 } dtp_status;
 
