@@ -81,7 +81,9 @@ class Clocks:
         self.path = None
 
     def __enter__(self):
-        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        # samples go to a git-ignored folder of the repository
+        os.makedirs(os.path.join(ROOT, "_build"), exist_ok=True)
+        fd, self.path = tempfile.mkstemp(suffix=".csv", prefix="clocks_", dir=os.path.join(ROOT, "_build"))
         os.close(fd)
         try:
             self.proc = subprocess.Popen(
