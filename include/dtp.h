@@ -116,11 +116,17 @@ int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate,
  *              points); n > 0: at most n CTAs, leaving the other SMs to
  *              kernels running concurrently on other streams (for instance the
  *              layout search of the previous layer, which runs on one SM)
+ *   flags      DTP_AFFINITY_DEFER_REDUCE: launch only the main kernel; its
+ *              per-unit partial sums stay in the workspace and
+ *              dtp_affinity_reduce adds them into A (and act2) later, possibly
+ *              on another stream (bf16 only)
  *   reserved   must be zero
  */
+#define DTP_AFFINITY_DEFER_REDUCE 1
 typedef struct dtp_affinity_opts {
     int max_ctas;
-    int reserved[7];
+    int flags;
+    int reserved[6];
 } dtp_affinity_opts;
 
 /*
@@ -133,6 +139,21 @@ int dtp_affinity_accumulate_opts(const void* X, const void* C, const void* W_gat
                                  const float* rms_next, int64_t T, int d, int H_kv, int N, int dtype,
                                  float* A, float* act2, const dtp_affinity_opts* opts, void* workspace,
                                  size_t workspace_bytes, void* stream);
+
+/*
+ * The second half of a deferred affinity pass: adds the workspace's per-unit
+ * partial sums into A [H_kv, N] (and, when act2 is non-NULL, the down-edge
+ * activation sums into act2 [N]), in the same fixed order as the undeferred
+ * call, so the result is bitwise the same.  T, d, H_kv, N and the workspace
+ * are those of the deferred call; the stream must be ordered after it (the
+ * caller records an event) and before the workspace is reused.
+ *   max_blocks  0: a grid over the whole GPU; n > 0: n blocks of 1024 threads,
+ *               for a reduce that runs beside a kernel holding the other SMs
+ *   overwrite   nonzero: A (and act2) receive the sums instead of adding them
+ *               (equal bit for bit to zeroing them first)
+ */
+int dtp_affinity_reduce(const void* workspace, size_t workspace_bytes, int64_t T, int d, int H_kv, int N,
+                        float* A, float* act2, int max_blocks, int overwrite, void* stream);
 
 /*
  * The first-order score per query head, summed over the query heads of each

@@ -411,7 +411,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
 constexpr int kReduceSplit = 8;
 __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
                                        int NT, int TC, const float* __restrict__ partial_act,
-                                       float* __restrict__ act2, int qpg) {
+                                       float* __restrict__ act2, int qpg, int overwrite) {
     const int64_t total_a = static_cast<int64_t>(G / qpg) * N;
     const int64_t total = total_a + (act2 ? N : 0);
     const int s = threadIdx.x % kReduceSplit;
@@ -436,9 +436,51 @@ __global__ void affinity_reduce_kernel(const float* __restrict__ partial, float*
         sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 2);
         sum += __shfl_xor_sync(0xFFFFFFFFu, sum, 1);
         if (s == 0) {
-            if (idx < total_a) A[idx] += sum;
-            else if (idx < total) act2[idx - total_a] += sum;
+            if (idx < total_a) A[idx] = overwrite ? sum : A[idx] + sum;
+            else if (idx < total) act2[idx - total_a] = overwrite ? sum : act2[idx - total_a] + sum;
         }
+    }
+}
+
+// The same sums with one thread per output, for a reduce confined to a few SMs: consecutive
+// threads take consecutive neurons, so each token chunk's loads are coalesced.  The thread keeps
+// the eight interleaved chunk sums c = s, s+8, ... (s = 0..7) that the eight threads of
+// affinity_reduce_kernel form and adds them by the same tree (s^4, then s^2, then s^1), so the
+// result is bitwise the same.
+__global__ void affinity_reduce_rows_kernel(const float* __restrict__ partial, float* __restrict__ A, int G, int N,
+                                            int NT, int TC, const float* __restrict__ partial_act,
+                                            float* __restrict__ act2, int qpg, int overwrite) {
+    const int64_t total_a = static_cast<int64_t>(G / qpg) * N;
+    const int64_t total = total_a + (act2 ? N : 0);
+    for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
+         idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        float acc[kReduceSplit];
+#pragma unroll
+        for (int s = 0; s < kReduceSplit; ++s) acc[s] = 0.0f;
+        if (idx < total_a) {
+            const int g = static_cast<int>(idx / N);
+            const int k = static_cast<int>(idx % N);
+            const int j = k / BNEU, r = k % BNEU;
+            for (int h = g * qpg; h < (g + 1) * qpg; ++h)
+                for (int c0 = 0; c0 < TC; c0 += kReduceSplit) {
+#pragma unroll
+                    for (int s = 0; s < kReduceSplit; ++s)
+                        if (c0 + s < TC)
+                            acc[s] += partial[((static_cast<int64_t>(c0 + s) * NT + j) * G + h) * BNEU + r];
+                }
+        } else {
+            const int k = static_cast<int>(idx - total_a);
+            const int j = k / BNEU, r = k % BNEU;
+            for (int c0 = 0; c0 < TC; c0 += kReduceSplit) {
+#pragma unroll
+                for (int s = 0; s < kReduceSplit; ++s)
+                    if (c0 + s < TC) acc[s] += partial_act[(static_cast<int64_t>(c0 + s) * NT + j) * BNEU + r];
+            }
+        }
+        // the tree of the shuffle reduction: lanes s and s^4, then s^2, then s^1
+        const float sum = ((acc[0] + acc[4]) + (acc[2] + acc[6])) + ((acc[1] + acc[5]) + (acc[3] + acc[7]));
+        if (idx < total_a) A[idx] = overwrite ? sum : A[idx] + sum;
+        else act2[idx - total_a] = overwrite ? sum : act2[idx - total_a] + sum;
     }
 }
 
@@ -488,11 +530,46 @@ size_t workspace_bytes_with_act(int64_t T, int d, int G, int N) {
     return align_up(workspace_bytes(T, d, G, N), 256) + static_cast<size_t>(NT * TC) * BNEU * sizeof(float);
 }
 
+// The fixed-order reduce of a workspace's unit partials into A (and act2 when the workspace
+// holds the down-edge activation sums): G heads in the workspace, G / qpg rows of A.
+// max_blocks > 0: that many blocks of 1024 threads (a reduce beside a kernel that holds every
+// other SM); overwrite: store the sums instead of adding them.
+int launch_reduce(const void* workspace, int64_t T, int d, int G, int N, float* A, float* act2, int qpg,
+                  cudaStream_t stream, int max_blocks, int overwrite) {
+    if (qpg < 1 || G % qpg) return DTP_ERR_ARG;
+    const int NT = (N + BNEU - 1) / BNEU;
+    const int TC = static_cast<int>((T + BT - 1) / BT);
+    const float* partial = reinterpret_cast<const float*>(reinterpret_cast<const uint8_t*>(workspace) +
+                                                          kWorkspaceHeader);
+    const float* partial_act = act2 ? reinterpret_cast<const float*>(reinterpret_cast<const uint8_t*>(workspace) +
+                                                                     align_up(workspace_bytes(T, d, G, N), 256))
+                                    : nullptr;
+    int dev = 0, sms = 0;
+    DTP_CUDA_TRY(cudaGetDevice(&dev));
+    DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const int64_t total = static_cast<int64_t>(G / qpg) * N + (act2 ? N : 0);
+    if (max_blocks > 0) {
+        const int64_t want = (total + 1023) / 1024;
+        const int rblocks = static_cast<int>(want < max_blocks ? want : max_blocks);
+        affinity_reduce_rows_kernel<<<rblocks, 1024, 0, stream>>>(partial, A, G, N, NT, TC, partial_act, act2, qpg,
+                                                                  overwrite);
+        DTP_CUDA_TRY(cudaGetLastError());
+        return DTP_OK;
+    }
+    const int64_t outs_per_block = 256 / kReduceSplit;
+    const int64_t want = (total + outs_per_block - 1) / outs_per_block;
+    const int rblocks = static_cast<int>(want < 8 * sms ? want : 8 * sms);
+    affinity_reduce_kernel<<<rblocks, 256, 0, stream>>>(partial, A, G, N, NT, TC, partial_act, act2, qpg, overwrite);
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
+}
+
 // G heads of C; A receives G / qpg rows (qpg consecutive heads summed per row).  max_ctas > 0
-// caps the persistent grid below one CTA per SM (leaving SMs to concurrent kernels).
+// caps the persistent grid below one CTA per SM (leaving SMs to concurrent kernels); with
+// defer_reduce the unit partials stay in the workspace for a later launch_reduce.
 int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N,
                    float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg,
-                   int max_ctas) {
+                   int max_ctas, int defer_reduce) {
     if (qpg < 1 || G % qpg) return DTP_ERR_ARG;
     CUtensorMap m_wg, m_wu, m_x, m_c;
     const cuuint64_t row_stride = static_cast<cuuint64_t>(d) * 2;
@@ -541,19 +618,13 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     p.tail_items = left * p.split;
     affinity_fo_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(m_wg, m_wu, m_x, m_c, p);
     DTP_CUDA_TRY(cudaGetLastError());
-    const int64_t total = static_cast<int64_t>(G / qpg) * N + (p.rms ? N : 0);
-    const int64_t outs_per_block = 256 / kReduceSplit;
-    const int64_t want = (total + outs_per_block - 1) / outs_per_block;
-    const int rblocks = static_cast<int>(want < 8 * sms ? want : 8 * sms);
-    affinity_reduce_kernel<<<rblocks, 256, 0, stream>>>(p.partial, A, G, N, p.NT, p.TC, p.partial_act,
-                                                        p.rms ? act2 : nullptr, qpg);
-    DTP_CUDA_TRY(cudaGetLastError());
-    return DTP_OK;
+    if (defer_reduce) return DTP_OK;
+    return launch_reduce(workspace, T, d, G, N, A, p.rms ? act2 : nullptr, qpg, stream, 0, 0);
 }
 
 int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N, float* A,
            void* workspace, cudaStream_t stream, const float* rms, float* act2) {
-    return launch_grouped(X, C, Wg, Wu, T, d, G, N, A, workspace, stream, rms, act2, 1, 0);
+    return launch_grouped(X, C, Wg, Wu, T, d, G, N, A, workspace, stream, rms, act2, 1, 0, 0);
 }
 
 }  // namespace tc

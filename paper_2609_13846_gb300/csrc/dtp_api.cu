@@ -13,7 +13,9 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
            void* workspace, cudaStream_t stream, const float* rms, float* act2);
 int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu, int64_t T, int d, int G, int N,
                    float* A, void* workspace, cudaStream_t stream, const float* rms, float* act2, int qpg,
-                   int max_ctas);
+                   int max_ctas, int defer_reduce);
+int launch_reduce(const void* workspace, int64_t T, int d, int G, int N, float* A, float* act2, int qpg,
+                  cudaStream_t stream, int max_blocks, int overwrite);
 }  // namespace tc
 namespace f32 {
 size_t workspace_bytes(int64_t T, int d, int G, int N);
@@ -155,10 +157,12 @@ int dtp_affinity_accumulate_opts(const void* X, const void* C, const void* W_gat
                                  const float* rms_next, int64_t T, int d, int H_kv, int N, int dtype, float* A,
                                  float* act2, const dtp_affinity_opts* opts, void* workspace, size_t workspace_bytes,
                                  void* stream) {
-    if (!opts || opts->max_ctas < 0) return DTP_ERR_ARG;
-    for (int i = 0; i < 7; ++i)
+    if (!opts || opts->max_ctas < 0 || (opts->flags & ~DTP_AFFINITY_DEFER_REDUCE)) return DTP_ERR_ARG;
+    for (int i = 0; i < 6; ++i)
         if (opts->reserved[i] != 0) return DTP_ERR_ARG;
-    if (dtype != DTP_BF16 || opts->max_ctas == 0)
+    const int defer = (opts->flags & DTP_AFFINITY_DEFER_REDUCE) != 0;
+    if (defer && dtype != DTP_BF16) return DTP_ERR_UNSUPPORTED;
+    if (dtype != DTP_BF16 || (opts->max_ctas == 0 && !defer))
         return dtp_affinity_accumulate_ex(X, C, W_gate, W_up, rms_next, T, d, H_kv, N, dtype, A, act2, workspace,
                                           workspace_bytes, stream);
     if (!affinity_sizes_ok(T, d, H_kv, N, dtype)) return DTP_ERR_ARG;
@@ -173,7 +177,19 @@ int dtp_affinity_accumulate_opts(const void* X, const void* C, const void* W_gat
         return DTP_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
-    return tc::launch_grouped(X, C, W_gate, W_up, T, d, H_kv, N, A, workspace, s, rms_next, act2, 1, opts->max_ctas);
+    return tc::launch_grouped(X, C, W_gate, W_up, T, d, H_kv, N, A, workspace, s, rms_next, act2, 1, opts->max_ctas,
+                              defer);
+}
+
+int dtp_affinity_reduce(const void* workspace, size_t workspace_bytes, int64_t T, int d, int H_kv, int N, float* A,
+                        float* act2, int max_blocks, int overwrite, void* stream) {
+    if (!affinity_sizes_ok(T, d, H_kv, N, DTP_BF16) || max_blocks < 0 || max_blocks > 65535) return DTP_ERR_ARG;
+    if (T == 0) return DTP_OK;
+    if (!A || !aligned16(A) || (act2 && !aligned16(act2))) return DTP_ERR_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < affinity_ws(T, d, H_kv, N, DTP_BF16, act2 != nullptr))
+        return DTP_ERR_WORKSPACE;
+    return tc::launch_reduce(workspace, T, d, H_kv, N, A, act2, 1, static_cast<cudaStream_t>(stream), max_blocks,
+                             overwrite ? 1 : 0);
 }
 
 int dtp_affinity_accumulate(const void* X, const void* C, const void* W_gate, const void* W_up, int64_t T, int d,
@@ -217,7 +233,7 @@ int dtp_affinity_accumulate_grouped(const void* X, const void* C_q, const void* 
         float* a2 = h0 == 0 ? act2 : nullptr;
         const int st = dtype == DTP_BF16
                            ? tc::launch_grouped(X, Cc, W_gate, W_up, T, d, hc, N, Ac, workspace, s, r, a2, q_per_group,
-                                                0)
+                                                0, 0)
                            : f32::launch_grouped(static_cast<const float*>(X), static_cast<const float*>(Cc),
                                                  static_cast<const float*>(W_gate), static_cast<const float*>(W_up), T,
                                                  d, hc, N, Ac, workspace, s, r, a2, q_per_group);

@@ -23,6 +23,7 @@ DTP_ERR_UNSUPPORTED = -4
 DTP_ERR_WORKSPACE = -5
 DTP_BF16 = 0
 DTP_F32 = 1
+DTP_AFFINITY_DEFER_REDUCE = 1
 
 _lib = None
 
@@ -34,7 +35,7 @@ _sz = ctypes.c_size_t
 
 class AffinityOpts(ctypes.Structure):
     """dtp_affinity_opts: max_ctas caps the persistent grid (0 = one CTA per SM)."""
-    _fields_ = [("max_ctas", ctypes.c_int), ("reserved", ctypes.c_int * 7)]
+    _fields_ = [("max_ctas", ctypes.c_int), ("flags", ctypes.c_int), ("reserved", ctypes.c_int * 6)]
 
 
 class DTPError(RuntimeError):
@@ -71,6 +72,7 @@ def lib():
                                                       _vp]
     L.dtp_affinity_accumulate_opts.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp,
                                                ctypes.POINTER(AffinityOpts), _vp, _sz, _vp]
+    L.dtp_affinity_reduce.argtypes = [_vp, _sz, _i64, _i32, _i32, _i32, _vp, _vp, _i32, _i32, _vp]
     L.dtp_affinity_add_workspace_size.argtypes = [_i64, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_affinity_add_accumulate.argtypes = [_vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
     L.dtp_down_weight_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
@@ -97,6 +99,7 @@ def lib():
                "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
                "dtp_head_writes_workspace_size", "dtp_head_writes", "dtp_layout_order", "dtp_permute_rows",
                "dtp_affinity_accumulate_opts", "dtp_search_global_workspace_size", "dtp_search_global",
+               "dtp_affinity_reduce",
                "dtp_permute_cols",
                "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
@@ -165,12 +168,13 @@ def affinity_workspace(T: int, d: int, H_kv: int, N: int, dtype: int, device) ->
 
 def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
                         A: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
-                        stream=None, max_ctas: int = 0) -> torch.Tensor:
+                        stream=None, max_ctas: int = 0, defer_reduce: bool = False) -> torch.Tensor:
     """A[h,k] += sum_t Delta_{t,h,k}^2 (Sec. 3); returns A [H_kv, N] fp32 on X's device.
 
     X [T,d], C [H_kv,T,d], W_gate/W_up [N,d]: contiguous CUDA tensors, all bf16
     or all fp32.  ``A`` is accumulated into (a zero tensor is made if None).
-    max_ctas > 0 caps the bf16 kernel's persistent grid (SMs left to other streams).
+    max_ctas > 0 caps the bf16 kernel's persistent grid (SMs left to other streams); with
+    defer_reduce only the main kernel runs and affinity_reduce(workspace, ...) finishes A later.
     """
     for name, t in (("X", X), ("C", C), ("W_gate", W_gate), ("W_up", W_up)):
         if not t.is_cuda or not t.is_contiguous():
@@ -189,8 +193,8 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
         raise ValueError("A must be a contiguous fp32 [H_kv, N] tensor on X's device")
     if workspace is None:
         workspace = affinity_workspace(T, d, H, N, code, X.device)
-    if max_ctas:
-        opts = AffinityOpts(max_ctas=int(max_ctas))
+    if max_ctas or defer_reduce:
+        opts = AffinityOpts(max_ctas=int(max_ctas), flags=DTP_AFFINITY_DEFER_REDUCE if defer_reduce else 0)
         st = lib().dtp_affinity_accumulate_opts(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), None, T, d, H, N, code,
                                                 _ptr(A), None, ctypes.byref(opts), _ptr(workspace), workspace.numel(),
                                                 _stream(stream))
@@ -199,6 +203,19 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
     st = lib().dtp_affinity_accumulate(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, code, _ptr(A),
                                        _ptr(workspace), workspace.numel(), _stream(stream))
     _check("dtp_affinity_accumulate", st)
+    return A
+
+
+def affinity_reduce(workspace: torch.Tensor, T: int, d: int, H_kv: int, N: int, A: torch.Tensor,
+                    act2: torch.Tensor | None = None, stream=None, max_blocks: int = 0,
+                    overwrite: bool = False) -> torch.Tensor:
+    """Add (or, with overwrite, store) the unit partials a deferred affinity pass left in
+    ``workspace`` into A (and act2); max_blocks > 0 runs it as that many 1024-thread blocks."""
+    if A.shape != (H_kv, N) or A.dtype != torch.float32 or not A.is_cuda or not A.is_contiguous():
+        raise ValueError("A must be a contiguous fp32 CUDA tensor [H_kv, N]")
+    st = lib().dtp_affinity_reduce(_ptr(workspace), workspace.numel(), T, d, H_kv, N, _ptr(A), _ptr(act2),
+                                   int(max_blocks), int(bool(overwrite)), _stream(stream))
+    _check("dtp_affinity_reduce", st)
     return A
 
 

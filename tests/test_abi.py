@@ -159,3 +159,18 @@ def test_global_search_size_rules(lib):
     assert lib.dtp_search_global_workspace_size(1, 16, 64, 2, ctypes.byref(n)) == 0      # 6435 partitions
     assert lib.dtp_search_global_workspace_size(1, 16, 64, 4, ctypes.byref(n)) == -1     # 2.6M partitions
     assert lib.dtp_search_global_workspace_size(1, 8, 30, 4, ctypes.byref(n)) == -1      # D does not divide N
+
+
+def test_affinity_defer_and_reduce_argument_checks(lib):
+    from paper_2609_13846_gb300 import dtp
+    buf = ctypes.create_string_buffer(1 << 12)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    bad = dtp.AffinityOpts(max_ctas=0, flags=2)                  # unknown flag
+    assert lib.dtp_affinity_accumulate_opts(p, p, p, p, None, 16, 64, 2, 128, 0, p, None, ctypes.byref(bad), p,
+                                            ctypes.c_size_t(1 << 12), None) == -1
+    f32 = dtp.AffinityOpts(max_ctas=0, flags=dtp.DTP_AFFINITY_DEFER_REDUCE)   # bf16 only
+    assert lib.dtp_affinity_accumulate_opts(p, p, p, p, None, 16, 64, 2, 128, 1, p, None, ctypes.byref(f32), p,
+                                            ctypes.c_size_t(1 << 12), None) == -4
+    assert lib.dtp_affinity_reduce(p, ctypes.c_size_t(16), 16, 64, 2, 128, p, None, 0, 0, None) == -5   # small ws
+    assert lib.dtp_affinity_reduce(p, ctypes.c_size_t(1 << 12), 16, 12, 2, 128, p, None, 0, 0, None) == -1  # d % 8
+    assert lib.dtp_affinity_reduce(p, ctypes.c_size_t(1 << 12), 16, 64, 2, 128, p, None, -1, 0, None) == -1

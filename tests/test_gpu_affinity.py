@@ -4,6 +4,8 @@ Tolerances (relative Frobenius error of A): 5e-3 for bf16 operands (tcgen05
 path), 1e-5 for the fp32 mode.  The inputs are the same bf16/fp32 values on
 both sides, so the error budget is fp32 accumulation and the fp32 epilogue.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -189,3 +191,45 @@ def test_full_model_layer_sampled_neurons_with_down_term(name):
     ref_act = oracle.down_activation(Lh["X"].double().numpy(), Lh["W_gate"][cols].double().numpy(),
                                      Lh["W_up"][cols].double().numpy(), Dn["rms"].double().cpu().numpy())
     assert _rel_fro(act2[torch.as_tensor(cols, device=DEV)].double().cpu().numpy(), ref_act) <= BF16_TOL
+
+
+@pytest.mark.parametrize("with_act", [False, True])
+def test_deferred_reduce_on_another_stream_is_bitwise_the_same(with_act):
+    """The main kernel alone (partials left in the workspace), then the reduce on a second
+    stream ordered by an event: A (and act2) equal the one-call result bit for bit."""
+    d, G, N, T = 512, 8, 640, 1000
+    L = synth.make_layer(d, G, N, T, seed=33, dtype="bf16")
+    g = {k: v.to(DEV) for k, v in L.items()}
+    rms = (0.5 + torch.rand(T, generator=torch.Generator().manual_seed(2))).to(DEV)
+    ws = dtp.affinity_workspace(T, d, G, N, dtp.DTP_BF16, DEV)
+    if with_act:
+        ref, ref_act = dtp.affinity_accumulate_down(g["X"], g["C"], g["W_gate"], g["W_up"], rms)
+    else:
+        ref = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"])
+    A = torch.zeros((G, N), dtype=torch.float32, device=DEV)
+    act2 = torch.zeros(N, dtype=torch.float32, device=DEV) if with_act else None
+    opts = dtp.AffinityOpts(max_ctas=100, flags=dtp.DTP_AFFINITY_DEFER_REDUCE)
+    st = dtp.lib().dtp_affinity_accumulate_opts(dtp._ptr(g["X"]), dtp._ptr(g["C"]), dtp._ptr(g["W_gate"]),
+                                                dtp._ptr(g["W_up"]), dtp._ptr(rms) if with_act else None, T, d, G,
+                                                N, dtp.DTP_BF16, dtp._ptr(A), dtp._ptr(act2), ctypes.byref(opts),
+                                                dtp._ptr(ws), ws.numel(), dtp._stream(None))
+    assert st == dtp.DTP_OK
+    assert not A.any()                                  # nothing reduced yet
+    ev = torch.cuda.Event()
+    ev.record()
+    side = torch.cuda.Stream()
+    side.wait_event(ev)
+    dtp.affinity_reduce(ws, T, d, G, N, A, act2, stream=side)
+    torch.cuda.synchronize()
+    assert torch.equal(A, ref)
+    if with_act:
+        assert torch.equal(act2, ref_act)
+    # the same partials reduced by one 1024-thread block, overwriting stale values
+    A.fill_(7.0)
+    if with_act:
+        act2.fill_(7.0)
+    dtp.affinity_reduce(ws, T, d, G, N, A, act2, max_blocks=1, overwrite=True)
+    torch.cuda.synchronize()
+    assert torch.equal(A, ref)
+    if with_act:
+        assert torch.equal(act2, ref_act)
