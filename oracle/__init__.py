@@ -47,7 +47,30 @@ def _load():
     global _lib
     if _lib is not None:
         return _lib
-    lib = ctypes.CDLL(build())
+    _lib = _declare(ctypes.CDLL(build()))
+    return _lib
+
+
+class use_library:
+    """Context manager: route every oracle call through another build of ``dtp_oracle.c`` (the
+    tests that plant a mistake in a copy of the source and check that a pin catches it)."""
+
+    def __init__(self, path: str):
+        self.path = path
+        self.saved = None
+
+    def __enter__(self):
+        global _lib
+        self.saved = _load()
+        _lib = _declare(ctypes.CDLL(self.path))
+        return self
+
+    def __exit__(self, *exc):
+        global _lib
+        _lib = self.saved
+
+
+def _declare(lib):
     lib.oracle_num_threads.restype = ctypes.c_int
     lib.oracle_affinity_fo.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int,
                                        ctypes.c_int, ctypes.c_int, _f64p]
@@ -105,7 +128,6 @@ def _load():
     lib.oracle_chain_edge_scores.argtypes = [_f32p, _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p,
                                              _i64p]
     lib.oracle_chain_edge_scores.restype = ctypes.c_int
-    _lib = lib
     return lib
 
 
