@@ -509,6 +509,30 @@ int dtp_permute_cols(const void* src, void* dst, int layers, int64_t rows, int64
                      int block_cols, const int32_t* perm, int64_t perm_layer_stride, void* workspace,
                      size_t workspace_bytes, void* stream);
 
+/*
+ * The whole layout application of Sec. 3 in one call: the orders of the head
+ * partitions and neuron assignments of `layers` layers, and the gathers of
+ * the seven weight matrices, stacked [layers, ...] in one element type:
+ *   src[0], dst[0]  q_proj  [layers, H_kv*q_per_group*head_dim, d]  (rows by KV group)
+ *   src[1], dst[1]  k_proj  [layers, H_kv*head_dim, d]               (rows by KV group)
+ *   src[2], dst[2]  v_proj  [layers, H_kv*head_dim, d]               (rows by KV group)
+ *   src[3], dst[3]  o_proj  [layers, d, H_kv*q_per_group*head_dim]   (columns by KV group)
+ *   src[4], dst[4]  gate_proj [layers, N, d]                         (rows by neuron)
+ *   src[5], dst[5]  up_proj   [layers, N, d]                         (rows by neuron)
+ *   src[6], dst[6]  down_proj [layers, d, N]                         (columns by neuron)
+ * src and dst are host arrays of 7 device pointers (dst distinct from src);
+ * head_part [layers, H_kv] and neuron_dev [layers, N] int32 device, balanced;
+ * head_order [layers, H_kv] and neuron_order [layers, N] int32 device out
+ * (dtp_layout_order's).  Device l's shard of the permuted weights is then the
+ * l-th contiguous slice.  Workspace: dtp_head_writes_workspace_size bytes;
+ * unbalanced layouts and labels outside [0, D) are reported through its status
+ * word.  Asynchronous; 9 launches.
+ */
+int dtp_apply_layout(const int32_t* head_part, const int32_t* neuron_dev, int layers, int H_kv, int N, int D,
+                     int q_per_group, int head_dim, int d, int elem_bytes, const void* const* src,
+                     void* const* dst, int32_t* head_order, int32_t* neuron_order, void* workspace,
+                     size_t workspace_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

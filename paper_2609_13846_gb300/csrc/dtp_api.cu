@@ -352,6 +352,40 @@ int dtp_permute_cols(const void* src, void* dst, int layers, int64_t rows, int64
                               elem_bytes, perm, perm_layer_stride, workspace, s);
 }
 
+int dtp_apply_layout(const int32_t* head_part, const int32_t* neuron_dev, int layers, int H_kv, int N, int D,
+                     int q_per_group, int head_dim, int d, int elem_bytes, const void* const* src, void* const* dst,
+                     int32_t* head_order, int32_t* neuron_order, void* workspace, size_t workspace_bytes,
+                     void* stream) {
+    if (layers < 1 || layers > 65535 || H_kv < 1 || N < 1 || D < 1 || H_kv % D || N % D || q_per_group < 1 ||
+        head_dim < 1 || d < 1 || elem_bytes < 1 || elem_bytes > 16)
+        return DTP_ERR_ARG;
+    if (!head_part || !neuron_dev || !src || !dst || !head_order || !neuron_order) return DTP_ERR_ARG;
+    for (int i = 0; i < 7; ++i)
+        if (!src[i] || !dst[i] || src[i] == dst[i]) return DTP_ERR_ARG;
+    if (!workspace || workspace_bytes < kWorkspaceHeader || !aligned16(workspace)) return DTP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DTP_CUDA_TRY(cudaMemsetAsync(workspace, 0, kWorkspaceHeader, s));
+    int st = apply::launch_order(head_part, layers, H_kv, D, 1, head_order, workspace, s);
+    if (st == DTP_OK) st = apply::launch_order(neuron_dev, layers, N, D, 1, neuron_order, workspace, s);
+    const int64_t qrows = static_cast<int64_t>(H_kv) * q_per_group * head_dim;   // q_proj rows, o_proj columns
+    const int64_t kvrows = static_cast<int64_t>(H_kv) * head_dim;
+    const int64_t row = static_cast<int64_t>(d) * elem_bytes;
+    const int qblk = q_per_group * head_dim;
+    // q, k, v rows and o columns by KV group; gate, up rows and down columns by neuron
+    if (st == DTP_OK) st = apply::launch_rows(src[0], dst[0], layers, qrows, row, qblk, head_order, H_kv, workspace, s);
+    if (st == DTP_OK) st = apply::launch_rows(src[1], dst[1], layers, kvrows, row, head_dim, head_order, H_kv, workspace, s);
+    if (st == DTP_OK) st = apply::launch_rows(src[2], dst[2], layers, kvrows, row, head_dim, head_order, H_kv, workspace, s);
+    if (st == DTP_OK)
+        st = apply::launch_cols(src[3], dst[3], layers, d, qrows * elem_bytes, static_cast<int64_t>(qblk) * elem_bytes,
+                                elem_bytes, head_order, H_kv, workspace, s);
+    if (st == DTP_OK) st = apply::launch_rows(src[4], dst[4], layers, N, row, 1, neuron_order, N, workspace, s);
+    if (st == DTP_OK) st = apply::launch_rows(src[5], dst[5], layers, N, row, 1, neuron_order, N, workspace, s);
+    if (st == DTP_OK)
+        st = apply::launch_cols(src[6], dst[6], layers, d, static_cast<int64_t>(N) * elem_bytes, elem_bytes,
+                                elem_bytes, neuron_order, N, workspace, s);
+    return st;
+}
+
 int dtp_down_weight_workspace_size(int H_kv, int R, int d, int N, size_t* bytes) {
     if (!bytes || H_kv < 1 || H_kv > kMaxHeads || R < 1 || d < 8 || (d % 8) || N < 1) return DTP_ERR_ARG;
     *bytes = sq::down_workspace_bytes(H_kv, R, d, N);

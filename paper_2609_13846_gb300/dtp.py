@@ -90,6 +90,8 @@ def lib():
     L.dtp_permute_cols.argtypes = [_vp, _vp, _i32, _i64, _i64, _i32, _i32, _vp, _i64, _vp, _sz, _vp]
     L.dtp_search_global_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_global.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+    L.dtp_apply_layout.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32,
+                                   ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp, _vp, _sz, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -99,7 +101,7 @@ def lib():
                "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
                "dtp_head_writes_workspace_size", "dtp_head_writes", "dtp_layout_order", "dtp_permute_rows",
                "dtp_affinity_accumulate_opts", "dtp_search_global_workspace_size", "dtp_search_global",
-               "dtp_affinity_reduce",
+               "dtp_affinity_reduce", "dtp_apply_layout",
                "dtp_permute_cols",
                "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
@@ -669,6 +671,30 @@ def apply_layout(W: dict, h: torch.Tensor, nu: torch.Tensor, D: int, head_dim: i
     h [layers, G] and nu [layers, N] then share.  Other entries are copied by
     reference.  Returns (permuted weights, head order, neuron order).
     """
+    names = ("q", "k", "v", "o", "gate", "up", "down")
+    mats = [W[n] for n in names]
+    stacked = h.dim() == 2
+    if all(m.is_cuda and m.is_contiguous() and m.dtype == mats[0].dtype and m.dim() == (3 if stacked else 2)
+           for m in mats) and h.dtype == torch.int32 and nu.dtype == torch.int32:
+        # one native call: both orders and the seven gathers
+        Lyr = h.shape[0] if stacked else 1
+        G, N, d = h.shape[-1], nu.shape[-1], mats[0].shape[-1]
+        qpg = mats[0].shape[-2] // (G * head_dim)
+        outs = [torch.empty_like(m) for m in mats]
+        hc, nc = _keep(h.contiguous(), stream), _keep(nu.contiguous(), stream)
+        ho, no = torch.empty_like(hc), torch.empty_like(nc)
+        ws = _status_workspace(h.device, stream)
+        src = (_vp * 7)(*[m.data_ptr() for m in mats])
+        dst = (_vp * 7)(*[o.data_ptr() for o in outs])
+        st = lib().dtp_apply_layout(_ptr(hc), _ptr(nc), Lyr, G, N, D, qpg, head_dim, d,
+                                    mats[0].element_size(), src, dst, _ptr(ho), _ptr(no), _ptr(ws), ws.numel(),
+                                    _stream(stream))
+        _check("dtp_apply_layout", st)
+        if check:
+            _check("dtp_apply_layout (device status)", workspace_status(ws, stream))
+        out = dict(W)
+        out.update(zip(names, outs))
+        return out, ho, no
     ho = layout_order(h, D, stream=stream, check=check)
     no = layout_order(nu, D, stream=stream, check=check)
     G = h.shape[-1]
