@@ -174,3 +174,17 @@ def test_affinity_defer_and_reduce_argument_checks(lib):
     assert lib.dtp_affinity_reduce(p, ctypes.c_size_t(16), 16, 64, 2, 128, p, None, 0, 0, None) == -5   # small ws
     assert lib.dtp_affinity_reduce(p, ctypes.c_size_t(1 << 12), 16, 12, 2, 128, p, None, 0, 0, None) == -1  # d % 8
     assert lib.dtp_affinity_reduce(p, ctypes.c_size_t(1 << 12), 16, 64, 2, 128, p, None, -1, 0, None) == -1
+
+
+def test_apply_layout_argument_checks(lib):
+    buf = ctypes.create_string_buffer(1 << 12)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    ptrs = (ctypes.c_void_p * 7)(*([p.value + 16 * i for i in range(7)]))
+    outs = (ctypes.c_void_p * 7)(*([p.value + 1024 + 16 * i for i in range(7)]))
+    same = (ctypes.c_void_p * 7)(*([p.value + 16 * i for i in range(7)]))
+    ws = ctypes.c_size_t(1 << 12)
+    # D does not divide the heads; a source used as its own destination; a null pointer array; no workspace
+    assert lib.dtp_apply_layout(p, p, 2, 8, 64, 3, 2, 16, 64, 2, ptrs, outs, p, p, p, ws, None) == -1
+    assert lib.dtp_apply_layout(p, p, 2, 8, 64, 4, 2, 16, 64, 2, ptrs, same, p, p, p, ws, None) == -1
+    assert lib.dtp_apply_layout(p, p, 2, 8, 64, 4, 2, 16, 64, 2, None, outs, p, p, p, ws, None) == -1
+    assert lib.dtp_apply_layout(p, p, 2, 8, 64, 4, 2, 16, 64, 2, ptrs, outs, p, p, None, ws, None) == -5
