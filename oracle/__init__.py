@@ -96,6 +96,8 @@ def _declare(lib):
     lib.oracle_global_layout.argtypes = [_f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _i32p, _i32p, _i64p,
                                          _f64p, _i32p]
     lib.oracle_global_layout.restype = ctypes.c_int
+    lib.oracle_top_group_share.argtypes = [_f32p, ctypes.c_int, ctypes.c_int]
+    lib.oracle_top_group_share.restype = ctypes.c_double
     lib.oracle_head_writes.argtypes = [_f64p, _f64p, _f64p, _f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
                                        ctypes.c_int, ctypes.c_int, _f64p]
     lib.oracle_head_writes.restype = None
@@ -438,3 +440,10 @@ def layout_order(labels, D: int) -> np.ndarray:
     if _load().oracle_layout_order(_p(lab, _i32p), lab.shape[0], D, _p(out, _i32p)) != 0:
         raise ValueError("label outside [0, D)")
     return out
+
+
+def top_group_share(A) -> float:
+    """Mean over neurons of max_g A[g,k] / sum_g A[g,k] (Sec. 5; neurons with a zero column skipped)."""
+    A = _c(A, np.float32)
+    G, N = A.shape
+    return float(_load().oracle_top_group_share(_p(A, _f32p), G, N))

@@ -869,6 +869,31 @@ int oracle_global_layout(const float* A, int G, int N, int D, int* h, int* nu, i
 }
 
 /* ------------------------------------------------------------------------ */
+/* Diagnostics                                                               */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Top-group share of a layer (Sec. 5, "Where the affinity concentrates"): for
+ * each neuron the largest KV group's fraction of its up-edge affinity,
+ * max_g A[g,k] / sum_g A[g,k], averaged over the neurons with a non-zero
+ * column (0 when there is none).  1/G when the groups contribute equally.
+ */
+double oracle_top_group_share(const float* A, int G, int N) {
+    double acc = 0.0;
+    int n = 0;
+    for (int k = 0; k < N; ++k) {
+        double tot = 0.0, mx = 0.0;
+        for (int g = 0; g < G; ++g) {
+            const double a = A[(int64_t)g * N + k];
+            tot += a;
+            if (a > mx) mx = a;
+        }
+        if (tot > 0.0) { acc += mx / tot; ++n; }
+    }
+    return n ? acc / n : 0.0;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Producer and layout application                                           */
 /* ------------------------------------------------------------------------ */
 

@@ -280,3 +280,20 @@ def test_more_than_sixteen_heads_equal_split_calls():
     np.testing.assert_array_equal(A, np.concatenate([oracle.affinity_fo(X, C[:16], Wg, Wu),
                                                      oracle.affinity_fo(X, C[16:], Wg, Wu)]))
     assert oracle.affinity_fo_qheads(X, C, Wg, Wu, 4).shape == (8, Wg.shape[0])
+
+
+def test_top_group_share_pins():
+    """Sec. 5: the largest KV group's share of a neuron's affinity, averaged over neurons."""
+    G, N = 8, 40
+    assert oracle.top_group_share(np.ones((G, N), np.float32)) == pytest.approx(1 / G, rel=1e-12)
+    one_hot = np.zeros((G, N), np.float32)
+    one_hot[np.arange(N) % G, np.arange(N)] = 3.0
+    assert oracle.top_group_share(one_hot) == pytest.approx(1.0, rel=1e-12)
+    A = np.zeros((2, 3), np.float32)
+    A[:, 0] = [1.0, 3.0]                        # 3/4
+    A[:, 2] = [2.0, 2.0]                        # 1/2; column 1 is empty and skipped
+    assert oracle.top_group_share(A) == pytest.approx((0.75 + 0.5) / 2, rel=1e-12)
+    assert oracle.top_group_share(np.zeros((2, 3), np.float32)) == 0.0
+    B = synth.make_affinity_matrix(G, N, seed=4).numpy()
+    assert oracle.top_group_share(B * np.float32(8.0)) == pytest.approx(oracle.top_group_share(B), rel=1e-12)
+    assert oracle.top_group_share(B[::-1].copy()) == pytest.approx(oracle.top_group_share(B), rel=1e-12)
