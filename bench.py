@@ -378,6 +378,7 @@ def run_model(args):
         torch.cuda.synchronize()
         searches[f"D{D}"] = {"ms": s0.elapsed_time(s1) / 3, "J": float(r["J"]), "J_random": (2 * Lyr - 1) / D,
                              "iters_done": int(r["iters_done"])}
+    share = dtp.top_group_share(S_up).cpu()              # Sec. 5: largest KV group's share per neuron
     suite, (h_opt, nu_opt, D_opt) = layout_suite(args, w, S_up, S_down, S_add if args.add_score else None, stream)
     apply = time_apply(w, h_opt, nu_opt, D_opt, stream)
     total_ms = t_aff + t_down + sum(v["ms"] for v in searches.values()) + t_prod + t_add + t_gather
@@ -392,6 +393,8 @@ def run_model(args):
             "affinity_ms": t_aff, "affinity_tflops": fl / (t_aff / 1e3) / 1e12,
             "layer_tokens_per_s": Lyr * T / (t_aff / 1e3), "down_edge_ms": t_down, "search": searches,
             "add_affinity_ms": t_add if args.add_score else None, "layout_suite": suite, "apply": apply,
+            "top_group_share": {"min": float(share.min()), "max": float(share.max()), "mean": float(share.mean()),
+                                "uniform": 1.0 / G},
             "pipeline_s": (total_ms + suite["ms"] + apply["ms"]) / 1e3,
             "producer_ms": t_prod if args.producer else None,
             "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s"}

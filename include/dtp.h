@@ -185,6 +185,17 @@ int dtp_affinity_accumulate_grouped(const void* X, const void* C_q, const void* 
                                     void* stream);
 
 /*
+ * Where a layer's affinity concentrates (Sec. 5): for each neuron the largest
+ * KV group's share of its column, max_g A[g,k] / sum_g A[g,k], averaged over
+ * the neurons whose column is not zero (0 when none is); 1/H_kv when the groups
+ * contribute equally.  fp64 arithmetic, fixed reduction order.
+ *   A      [layers, H_kv, N] fp32, device, entries finite and >= 0
+ *   share  [layers] double out, device
+ * Asynchronous; no workspace.
+ */
+int dtp_affinity_top_share(const float* A, int layers, int H_kv, int N, double* share, void* stream);
+
+/*
  * The ADD score of Sec. 3 before the mean: the squared additive contribution
  * of KV group h's piece to neuron k's pre-activations, ignoring the operating
  * point and ||w^d_k||:

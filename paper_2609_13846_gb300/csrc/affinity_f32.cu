@@ -238,6 +238,50 @@ int launch_down_finalize(const float* act2, const float* bn, int G, int N, int64
     return DTP_OK;
 }
 
+// Top-group share of each layer (Sec. 5 diagnostic): the mean over neurons with a non-zero column of
+// max_g A[g,k] / sum_g A[g,k], in fp64.  One block per layer; the per-thread sums are combined in a
+// fixed order (warp butterflies, then the warps in index order), so the result is reproducible.
+__global__ void __launch_bounds__(1024) top_share_kernel(const float* __restrict__ A, int G, int N,
+                                                         double* __restrict__ share) {
+    __shared__ double ssum[32];
+    __shared__ int scnt[32];
+    const float* a = A + static_cast<int64_t>(blockIdx.x) * G * N;
+    double acc = 0.0;
+    int cnt = 0;
+    for (int k = threadIdx.x; k < N; k += blockDim.x) {
+        double tot = 0.0, mx = 0.0;
+        for (int g = 0; g < G; ++g) {
+            const double v = a[static_cast<int64_t>(g) * N + k];
+            tot += v;
+            mx = v > mx ? v : mx;
+        }
+        if (tot > 0.0) {
+            acc += mx / tot;
+            ++cnt;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+        cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) ssum[warp] = acc, scnt[warp] = cnt;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        int c = 0;
+        for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += ssum[w], c += scnt[w];
+        share[blockIdx.x] = c ? t / c : 0.0;
+    }
+}
+
+int launch_top_share(const float* A, int layers, int G, int N, double* share, cudaStream_t stream) {
+    top_share_kernel<<<layers, 1024, 0, stream>>>(A, G, N, share);
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
+}
+
 int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream) {
     const int64_t total = static_cast<int64_t>(G) * N;
     const int blocks = static_cast<int>((total + 255) / 256 < 1024 ? (total + 255) / 256 : 1024);

@@ -47,6 +47,7 @@ int launch_cols(const void* src, void* dst, int layers, int64_t rows, int64_t ro
                 int elem_bytes, const int32_t* perm, int64_t perm_stride, void* workspace, cudaStream_t stream);
 }  // namespace apply
 int launch_finalize(float* A, int G, int N, int64_t T_total, const float* wd, cudaStream_t stream);
+int launch_top_share(const float* A, int layers, int G, int N, double* share, cudaStream_t stream);
 int launch_down_finalize(const float* act2, const float* bn, int G, int N, int64_t T_total, float* S,
                          cudaStream_t stream);
 int launch_down_sqnorm(const void* W, int d, int N, int dtype, float* out, cudaStream_t stream);
@@ -384,6 +385,13 @@ int dtp_apply_layout(const int32_t* head_part, const int32_t* neuron_dev, int la
         st = apply::launch_cols(src[6], dst[6], layers, d, static_cast<int64_t>(N) * elem_bytes, elem_bytes,
                                 elem_bytes, neuron_order, N, workspace, s);
     return st;
+}
+
+int dtp_affinity_top_share(const float* A, int layers, int H_kv, int N, double* share, void* stream) {
+    if (layers < 1 || layers > 65535 || H_kv < 1 || H_kv > kMaxHeads || N < 1) return DTP_ERR_ARG;
+    if (!A || !share || (reinterpret_cast<uintptr_t>(A) & 3) || (reinterpret_cast<uintptr_t>(share) & 7))
+        return DTP_ERR_ARG;
+    return launch_top_share(A, layers, H_kv, N, share, static_cast<cudaStream_t>(stream));
 }
 
 int dtp_down_weight_workspace_size(int H_kv, int R, int d, int N, size_t* bytes) {

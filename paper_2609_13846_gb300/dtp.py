@@ -92,6 +92,7 @@ def lib():
     L.dtp_search_global.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_apply_layout.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32,
                                    ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp, _vp, _sz, _vp]
+    L.dtp_affinity_top_share.argtypes = [_vp, _i32, _i32, _i32, _vp, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -101,7 +102,7 @@ def lib():
                "dtp_affinity_grouped_workspace_size", "dtp_affinity_accumulate_grouped",
                "dtp_head_writes_workspace_size", "dtp_head_writes", "dtp_layout_order", "dtp_permute_rows",
                "dtp_affinity_accumulate_opts", "dtp_search_global_workspace_size", "dtp_search_global",
-               "dtp_affinity_reduce", "dtp_apply_layout",
+               "dtp_affinity_reduce", "dtp_apply_layout", "dtp_affinity_top_share",
                "dtp_permute_cols",
                "dtp_affinity_add_grouped_workspace_size", "dtp_affinity_add_accumulate_grouped",
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
@@ -206,6 +207,18 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
                                        _ptr(workspace), workspace.numel(), _stream(stream))
     _check("dtp_affinity_accumulate", st)
     return A
+
+
+def top_group_share(A: torch.Tensor, stream=None) -> torch.Tensor:
+    """Mean over neurons of the largest KV group's share of the neuron's affinity (Sec. 5), per layer.
+    A [L, H_kv, N] (or [H_kv, N]) fp32 CUDA; returns float64 [L] (or a scalar)."""
+    x = A.unsqueeze(0) if A.dim() == 2 else A
+    if x.dtype != torch.float32 or not x.is_cuda or not x.is_contiguous():
+        raise ValueError("A must be a contiguous fp32 CUDA tensor")
+    out = _keep(torch.empty(x.shape[0], dtype=torch.float64, device=x.device), stream)
+    _check("dtp_affinity_top_share", lib().dtp_affinity_top_share(_ptr(x), x.shape[0], x.shape[1], x.shape[2],
+                                                                  _ptr(out), _stream(stream)))
+    return out if A.dim() == 3 else out[0]
 
 
 def affinity_reduce(workspace: torch.Tensor, T: int, d: int, H_kv: int, N: int, A: torch.Tensor,

@@ -233,3 +233,19 @@ def test_deferred_reduce_on_another_stream_is_bitwise_the_same(with_act):
     assert torch.equal(A, ref)
     if with_act:
         assert torch.equal(act2, ref_act)
+
+
+def test_top_group_share_matches_oracle():
+    mats = [synth.make_affinity_matrix(8, 3072, seed=s).numpy() for s in range(3)]
+    mats.append(np.ones((8, 3072), np.float32))
+    z = np.zeros((8, 3072), np.float32)
+    z[:, ::3] = synth.make_affinity_matrix(8, 1024, seed=9).numpy()
+    mats.append(z)                                      # two thirds of the columns empty
+    A = torch.as_tensor(np.stack(mats), device=DEV)
+    got = dtp.top_group_share(A).cpu().numpy()
+    for i, m in enumerate(mats):
+        assert got[i] == pytest.approx(oracle.top_group_share(m), rel=1e-12)
+    w = synth.WORKLOADS["qwen3_0.6b_layer"]
+    L = synth.make_workload_layer(w, T=2048, device=DEV)
+    Aw = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"])
+    assert float(dtp.top_group_share(Aw)) == pytest.approx(oracle.top_group_share(Aw.cpu().numpy()), rel=1e-12)
