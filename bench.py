@@ -444,8 +444,9 @@ def main():
     stream = torch.cuda.current_stream()
     side = torch.cuda.Stream(device=dev)
     n_sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    # Step pipeline: the affinity pass of step k runs on all SMs but one (max_ctas) while the
-    # layout search of step k-1 (one thread block) runs on the spare SM from a second stream.
+    # Step pipeline: the affinity pass of step k runs on all SMs but one (max_ctas; for this layer
+    # its CTA pairs round that down to 150 of 152) while the layout search of step k-1 (one thread
+    # block) runs on a spare SM from a second stream.
     # A and the search workspace are double-buffered; events order each buffer's reuse.  (Moving
     # the 12 us partial-sum reduce to the second stream as well measured slower.)
     A_buf = [torch.zeros((w.G, w.N), dtype=torch.float32, device=dev) for _ in range(2)]

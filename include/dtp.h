@@ -115,7 +115,10 @@ int dtp_affinity_accumulate_ex(const void* X, const void* C, const void* W_gate,
  *   max_ctas   0: one persistent CTA per SM (the default of the other entry
  *              points); n > 0: at most n CTAs, leaving the other SMs to
  *              kernels running concurrently on other streams (for instance the
- *              layout search of the previous layer, which runs on one SM)
+ *              layout search of the previous layer, which runs on one SM).
+ *              When the layer's W_gate and W_up fit in half of the L2 cache
+ *              the kernel runs as pairs of CTAs, and n is then rounded down
+ *              to an even count (at least one pair: 2 CTAs for n = 1)
  *   flags      DTP_AFFINITY_DEFER_REDUCE: launch only the main kernel; its
  *              per-unit partial sums stay in the workspace and
  *              dtp_affinity_reduce adds them into A (and act2) later, possibly
@@ -279,8 +282,9 @@ int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, voi
  * (bf16 inputs only), minus the workspace.  Scratch comes from one fixed
  * device array of 16 MiB + 256 B inside the library, present on every GPU
  * that loads it until the process exits; the call allocates nothing.
- *   - Limit: ceil(T/128) * ceil(N/128) * H_kv <= 32768 per call, else
- *     DTP_ERR_WORKSPACE (stream longer inputs as token chunks; A accumulates).
+ *   - Limit: c * ceil(N/128) * H_kv <= 32768 per call, with c = ceil(T/128)
+ *     rounded up to an even count, else DTP_ERR_WORKSPACE (stream longer
+ *     inputs as token chunks; A accumulates).
  *   - Every call shares the array and it keeps the last call's contents:
  *     calls that overlap on the GPU race and must be serialised by the caller.
  *   - The first call on a device looks up the array's device address with

@@ -34,7 +34,9 @@ int launch(const void* X, const void* C, const void* Wg, const void* Wu, int64_t
 }  // namespace dtp
 
 // 256-byte status header + 16 MiB of partial sums (512 B per token chunk,
-// neuron tile and head): ceil(T/128) * ceil(N/128) * H_kv <= 32768 per call.
+// neuron tile and head): c * ceil(N/128) * H_kv <= 32768 per call, c the
+// token-chunk count ceil(T/128) rounded up to an even count (the kernel's CTA
+// pairs take chunks two at a time).
 static constexpr int64_t kNoAllocMaxUnitHeads = 32768;
 static constexpr size_t kNoAllocScratchBytes = dtp::kWorkspaceHeader + (size_t(16) << 20);
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
@@ -73,7 +75,7 @@ extern "C" int dtp_affinity_accumulate_noalloc(const void* X, const void* C, con
     if (!dtp::aligned16(X) || !dtp::aligned16(C) || !dtp::aligned16(W_gate) || !dtp::aligned16(W_up) ||
         !dtp::aligned16(A))
         return DTP_ERR_ARG;
-    const int64_t unit_heads = ((T + 127) / 128) * ((static_cast<int64_t>(N) + 127) / 128) * H_kv;
+    const int64_t unit_heads = ((T + 255) / 256) * 2 * ((static_cast<int64_t>(N) + 127) / 128) * H_kv;
     if (unit_heads > kNoAllocMaxUnitHeads || dtp::tc::workspace_bytes(T, d, H_kv, N) > kNoAllocScratchBytes)
         return DTP_ERR_WORKSPACE;
     void* scratch = nullptr;

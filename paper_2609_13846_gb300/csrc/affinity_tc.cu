@@ -6,23 +6,43 @@
 // with g = X W_gate^T, u = X W_up^T (the operating point) and pg = C_h W_gate^T,
 // pu = C_h W_up^T (head h's piece projected through the FFN input weights).
 //
-// MMA shape.  One tcgen05.mma per 16-wide K step computes a 128-token x
-// 256-column tile: A = 128 rows of one activation tile (X or C_h), B = the
-// neuron tile's 128 W_gate rows stacked on its 128 W_up rows, so columns
-// [0,128) of the accumulator are g (or pg) and [128,256) are u (or pu) of the
-// same 128 neurons.  The kernel is bound by the number of MMA instructions it
-// issues, so the widest single-CTA instruction (N = 256) is used.
+// MMA shape, two forms of one kernel (template parameter kPair):
+//  - CTA pairs (clusters of two) sharing one tcgen05.mma of cta_group::2 per
+//    16-wide K step: M = 256 tokens (128 token rows of one activation tile,
+//    X or C_h, in each CTA), N = 256 columns (the neuron tile's 128 W_gate
+//    rows in the even CTA, its 128 W_up rows in the odd CTA).  Each SM stages
+//    and reads only half of the weight operand, which keeps the tensor pipe
+//    busier than a single-CTA instruction does.  Used when the weights fit in
+//    L2 with room to spare.
+//  - single CTAs issuing one tcgen05.mma of cta_group::1 per K step: M = 128
+//    tokens, N = 256 (W_gate and W_up tiles stacked).  Used for layers whose
+//    weights do not fit in L2: there the pairs' placement (a cluster's CTAs
+//    land on neighbouring SMs, consecutive clusters fill one part of the chip
+//    after another) cost the chunk grouping below most of its L2 reuse --
+//    several times the DRAM traffic on a Llama-3.1-8B-shaped layer.
+// In both, columns [0,128) of a CTA's accumulator are g (or pg) and [128,256)
+// are u (or pu) of the same 128 neurons for that CTA's 128 tokens.
 //
-// Work unit = (token chunk c of 128 tokens, neuron tile j of 128 neurons).  A
-// unit runs G+1 passes over d: pass 0 multiplies the X chunk, pass 1+h the C_h
-// chunk.  Units are dealt round-robin to a persistent grid in
-// token-chunk-major order, so the CTAs in flight share a handful of token
-// chunks in L2 while all weights stay L2-resident.  When the weights do not
-// fit in L2, token chunks are taken in groups and each neuron tile meets the
-// group's chunks back to back, so the units in flight share fewer weight
-// tiles.  The units left over after
-// the last full round are split by heads over several CTAs (each recomputes
-// the unit's X pass), so the final round keeps most SMs busy.
+// Work unit = (chunk unit, neuron tile j of 128 neurons); a chunk unit is a
+// pair of 128-token chunks (2 cu for the even CTA, 2 cu + 1 for the odd one)
+// in the pair form and one chunk in the single form.  A unit runs G+1 passes
+// over d: pass 0 multiplies the X chunks, pass 1+h the C_h chunks.  Units are
+// dealt round-robin to a persistent grid in chunk-unit-major order, so the
+// units in flight share a handful of token chunks in L2 while all weights
+// stay L2-resident.  When the weights do not fit in L2, chunk units are taken
+// in groups and each neuron tile meets the group's chunk units back to back,
+// so the units in flight share fewer weight tiles.  The units left over after
+// the last full round are split by heads over several workers (each
+// recomputes the unit's X pass), so the final round keeps most SMs busy.  In
+// the pair form with an odd chunk count, the odd CTA of the last pair reloads
+// the last chunk and stores its sums into a spare slot the reduce never reads.
+//
+// Pair protocol.  Both CTAs' TMA loads of a stage complete on the even CTA's
+// full barrier (one expect-tx of both CTAs' bytes); the even CTA's single MMA
+// thread waits there, issues the pair MMAs and commits to the empty barriers
+// and accumulator barriers of both CTAs at once (multicast); the epilogue
+// warps of both CTAs release an accumulator buffer by arriving on the even
+// CTA's barrier.
 //
 // TMEM (512 columns x 128 lanes = tokens, fp32): two accumulator buffers of
 // 256 columns used by passes alternately, so the epilogue of one pass
@@ -43,13 +63,17 @@
 // over tokens per neuron -- E_t[alpha_k^2 / r'^2] of the down-edge score before
 // the mean -- with the same butterfly and quadrant reduction.
 //
-// Warp roles (384 threads, 3 warpgroups): warp 0 issues TMA loads, warp 1
-// allocates TMEM and issues the MMAs (one thread), warps 2-3 idle; warpgroup
-// 0 gives registers back (setmaxnreg) to warpgroups 1-2, the epilogue.
+// Warp roles (384 threads, 3 warpgroups per CTA): warp 0 issues TMA loads,
+// warp 1 allocates TMEM (for the pair in the pair form) and issues the MMAs
+// (one thread; in the pair form only in the even CTA), warps 2-3 idle;
+// warpgroup 0 gives registers back (setmaxnreg) to warpgroups 1-2, the
+// epilogue.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <atomic>
 
 #include "dtp_common.cuh"
 
@@ -60,32 +84,40 @@ constexpr int BT = 128;       // tokens per chunk (MMA M, TMEM lanes)
 constexpr int BNEU = 128;     // neurons per tile (MMA N = 2 * BNEU: gate | up)
 constexpr int BK = 64;        // bf16 elements per 128-byte swizzled row
 constexpr int UK = 16;        // K of one tcgen05.mma kind::f16
-constexpr int STAGES = 4;
 constexpr int kThreads = 384;
 constexpr int kEpiWarps = 8;
 constexpr int kEpiWarp0 = 4;  // first epilogue warp
 constexpr uint32_t kRegsSmall = 56;   // warpgroup 0 after setmaxnreg.dec
 constexpr uint32_t kRegsLarge = 224;  // epilogue warpgroups after setmaxnreg.inc
 static_assert(128 * kRegsSmall + 256 * kRegsLarge <= kThreads * 168, "register split exceeds the launch budget");
-constexpr uint32_t kTileAct = BT * BK * 2;     // 16 KB activation operand (A)
-constexpr uint32_t kTileW = BNEU * BK * 2;     // 16 KB, W_gate or W_up half of B
-constexpr uint32_t kStageBytes = kTileAct + 2 * kTileW;
+constexpr uint32_t kTileAct = BT * BK * 2;     // 16 KB activation operand (this CTA's A rows)
+constexpr uint32_t kTileW = BNEU * BK * 2;     // 16 KB: the W_gate or the W_up rows of a neuron tile
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kBufCols = 256;
 constexpr size_t kRedBytes = 2 * 4 * BNEU * sizeof(float);   // [slot][quadrant][neuron]
-constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + kRedBytes + 256;
-constexpr uint32_t kIdesc = idesc_bf16_f32(BT, 2 * BNEU);
+
+// Per form: a stage holds this CTA's activation tile and its weight rows (half of B in the pair
+// form, both halves in the single form); both forms keep 192 KB of stages in flight.
+template <bool kPair>
+struct Form {
+    static constexpr int STAGES = kPair ? 6 : 4;
+    static constexpr uint32_t kStageBytes = kTileAct + (kPair ? 1u : 2u) * kTileW;
+    static constexpr uint32_t kIdesc = idesc_bf16_f32(kPair ? 2 * BT : BT, 2 * BNEU);
+    static constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + kRedBytes + 256;
+};
+static_assert(Form<true>::kSmemBytes <= 227 * 1024 && Form<false>::kSmemBytes <= 227 * 1024, "shared memory");
 
 struct Params {
     int G;            // KV heads
     int NT;           // neuron tiles
     int TC;           // token chunks
+    int TU;           // chunk units: chunk pairs ceil(TC / 2) (pair form) or chunks (single form)
     int KB;           // k blocks of 64 over d
-    int64_t units;    // NT * TC
-    int full_rounds;  // rounds in which every CTA takes one whole unit
+    int64_t units;    // NT * TU
+    int full_rounds;  // rounds in which every worker (CTA pair or CTA) takes one whole unit
     int split;        // head groups per left-over unit
-    int tail_items;   // left-over units * split (<= grid)
-    int cg;           // token chunks per group of the unit order (1 = chunk-major)
+    int tail_items;   // left-over units * split (<= workers)
+    int cg;           // chunk units per group of the unit order (1 = chunk-unit-major)
     int64_t T;        // tokens
     float* partial;   // [units][G][128]
     const float* rms; // [T] rms of the next layer's pre-norm input, or null
@@ -93,34 +125,39 @@ struct Params {
     int* status;      // workspace status word
 };
 
-// The i-th work item of this CTA: a unit and the head range [h0, h1) it covers.
+// The i-th work item of a worker (a CTA pair or a CTA): a unit and the head range [h0, h1) it covers.
 struct Item {
     int64_t unit;
     int h0, h1;
 };
 
-// Unit u in the processing order -> (token chunk c, neuron tile j).
-__device__ __forceinline__ void unit_coords(const Params& p, int64_t u, int& c, int& j) {
+// Unit u in the processing order -> (chunk unit cu, neuron tile j).  The chunk of a CTA is
+// 2 cu + (its rank in the pair) in the pair form and cu in the single form.
+__device__ __forceinline__ void unit_coords(const Params& p, int64_t u, int& cu, int& j) {
     const int64_t per_group = static_cast<int64_t>(p.cg) * p.NT;
     const int64_t grp = u / per_group;
     const int64_t r = u - grp * per_group;
     const int c0 = static_cast<int>(grp) * p.cg;
-    const int cn = p.TC - c0 < p.cg ? p.TC - c0 : p.cg;   // chunks in this (possibly last) group
+    const int cn = p.TU - c0 < p.cg ? p.TU - c0 : p.cg;   // chunk units in this (possibly last) group
     j = static_cast<int>(r / cn);
-    c = c0 + static_cast<int>(r % cn);
+    cu = c0 + static_cast<int>(r % cn);
 }
 
+// Workers: CTA pairs (clusters of two, blocks 2q and 2q + 1 form pair q) or single CTAs.
+template <bool kPair>
 __device__ __forceinline__ bool get_item(const Params& p, int i, Item& it) {
+    const int worker = static_cast<int>(kPair ? blockIdx.x >> 1 : blockIdx.x);
+    const int workers = static_cast<int>(kPair ? gridDim.x >> 1 : gridDim.x);
     if (i < p.full_rounds) {
-        it.unit = static_cast<int64_t>(i) * gridDim.x + blockIdx.x;
+        it.unit = static_cast<int64_t>(i) * workers + worker;
         it.h0 = 0;
         it.h1 = p.G;
         return true;
     }
-    if (i == p.full_rounds && static_cast<int>(blockIdx.x) < p.tail_items) {
-        const int t = static_cast<int>(blockIdx.x);
+    if (i == p.full_rounds && worker < p.tail_items) {
+        const int t = worker;
         const int grp = t % p.split;
-        it.unit = static_cast<int64_t>(p.full_rounds) * gridDim.x + t / p.split;
+        it.unit = static_cast<int64_t>(p.full_rounds) * workers + t / p.split;
         it.h0 = p.G * grp / p.split;
         it.h1 = p.G * (grp + 1) / p.split;
         return true;
@@ -146,27 +183,36 @@ __device__ __forceinline__ float butterfly32(float (&v)[32], int lane) {
     return v[0];
 }
 
+template <bool kPair>
 __global__ void __launch_bounds__(kThreads, 1)
 affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_constant__ CUtensorMap tm_wu,
                       const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_c,
                       const Params p) {
+    constexpr int STAGES = Form<kPair>::STAGES;
+    constexpr uint32_t kStageBytes = Form<kPair>::kStageBytes;
+    constexpr uint32_t kIdesc = Form<kPair>::kIdesc;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* tiles = smem;
     float* red = reinterpret_cast<float*>(smem + STAGES * kStageBytes);   // [2][4][128]
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes + kRedBytes);
-    // full[S], empty[S], acc_full[2], acc_empty[2], red_full[2], drain
+    // full[S], empty[S], acc_full[2], acc_empty[2], red_full[2], red_empty[2], drain.  In the pair
+    // form full and acc_empty are used in the even CTA only (both CTAs' loads and epilogues arrive
+    // there); empty, acc_full and drain receive the even CTA's commits in both CTAs.
     uint64_t* full_bar = bars;
     uint64_t* empty_bar = bars + STAGES;
     uint64_t* acc_full = bars + 2 * STAGES;
     uint64_t* acc_empty = acc_full + 2;
     uint64_t* red_full = acc_full + 4;
-    uint64_t* drain_bar = acc_full + 6;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 7);
+    uint64_t* red_empty = acc_full + 6;
+    uint64_t* drain_bar = acc_full + 8;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 9);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    const uint32_t rank = kPair ? cluster_ctarank() : 0u;   // 0: issues the MMAs; 1: its peer
+    const bool leader = rank == 0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -175,112 +221,134 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
-            mbar_init(smem_u32(&acc_empty[b]), kEpiWarps);
+            mbar_init(smem_u32(&acc_empty[b]), (kPair ? 2 : 1) * kEpiWarps);
             mbar_init(smem_u32(&red_full[b]), kEpiWarps);
+            mbar_init(smem_u32(&red_empty[b]), 2);   // the two summing warps
         }
         mbar_init(smem_u32(drain_bar), 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&tm_wg);
-        tma_prefetch_desc(&tm_wu);
+        if (!kPair || leader) tma_prefetch_desc(&tm_wg);
+        if (!kPair || !leader) tma_prefetch_desc(&tm_wu);
         tma_prefetch_desc(&tm_x);
         tma_prefetch_desc(&tm_c);
     }
     if (warp == 1) {
-        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
-        tmem_relinquish();
+        if constexpr (kPair) {
+            tmem_alloc_pair(smem_u32(tmem_slot), kTmemCols);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
-    __syncthreads();
+    if constexpr (kPair)
+        cluster_sync();   // both CTAs' barriers initialised and TMEM allocated before any remote access
+    else
+        __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
     if (warp < kEpiWarp0) {
         setmaxnreg_dec<kRegsSmall>();
         if (warp == 0 && lane == 0) {
-            // ---------------------------------------------------------------- producer
+            // ---------------------------------------------------------------- producer (every CTA)
+            const uint32_t full_lead = kPair ? mapa_shared(smem_u32(full_bar), 0) : 0u;   // the even CTA's full[0]
             int stage = 0;
             uint32_t phase = 0;
-            uint32_t issued_parity[STAGES];
-            bool issued[STAGES];
-            for (int s = 0; s < STAGES; ++s) issued[s] = false, issued_parity[s] = 0;
             bool ok = true;
             Item it;
-            for (int i = 0; ok && get_item(p, i, it); ++i) {
-                int c, j;
-                unit_coords(p, it.unit, c, j);
+            for (int i = 0; ok && get_item<kPair>(p, i, it); ++i) {
+                int cu, j;
+                unit_coords(p, it.unit, cu, j);
+                // the odd CTA of a last, half-empty pair reloads the last chunk (its sums go to a spare slot)
+                const int c_raw = kPair ? 2 * cu + static_cast<int>(rank) : cu;
+                const int c = c_raw < p.TC ? c_raw : p.TC - 1;
                 const int passes = 1 + it.h1 - it.h0;
                 for (int pass = 0; ok && pass < passes; ++pass) {
                     for (int kb = 0; kb < p.KB; ++kb) {
                         if (!mbar_wait(smem_u32(&empty_bar[stage]), phase ^ 1u, abort_flag)) { ok = false; break; }
-                        const uint32_t fb = smem_u32(&full_bar[stage]);
                         uint8_t* st = tiles + stage * kStageBytes;
-                        mbar_arrive_expect_tx(fb, kStageBytes);
-                        if (pass == 0)
-                            tma_load_2d(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
-                        else
-                            tma_load_3d(smem_u32(st), &tm_c, fb, kb * BK, c * BT, it.h0 + pass - 1);
-                        tma_load_2d(smem_u32(st + kTileAct), &tm_wg, fb, kb * BK, j * BNEU);
-                        tma_load_2d(smem_u32(st + kTileAct + kTileW), &tm_wu, fb, kb * BK, j * BNEU);
-                        issued[stage] = true;
-                        issued_parity[stage] = phase;
+                        if constexpr (kPair) {
+                            const uint32_t fb = full_lead + static_cast<uint32_t>(stage) * 8u;
+                            if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[stage]), 2 * kStageBytes);
+                            if (pass == 0)
+                                tma_load_2d_pair(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
+                            else
+                                tma_load_3d_pair(smem_u32(st), &tm_c, fb, kb * BK, c * BT, it.h0 + pass - 1);
+                            tma_load_2d_pair(smem_u32(st + kTileAct), leader ? &tm_wg : &tm_wu, fb, kb * BK, j * BNEU);
+                        } else {
+                            const uint32_t fb = smem_u32(&full_bar[stage]);
+                            mbar_arrive_expect_tx(fb, kStageBytes);
+                            if (pass == 0)
+                                tma_load_2d(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
+                            else
+                                tma_load_3d(smem_u32(st), &tm_c, fb, kb * BK, c * BT, it.h0 + pass - 1);
+                            tma_load_2d(smem_u32(st + kTileAct), &tm_wg, fb, kb * BK, j * BNEU);
+                            tma_load_2d(smem_u32(st + kTileAct + kTileW), &tm_wu, fb, kb * BK, j * BNEU);
+                        }
                         if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                     }
                 }
             }
-            if (!ok) {
-                // Let copies already in flight land before the CTA exits.
-                for (int s = 0; s < STAGES; ++s)
-                    if (issued[s]) {
-                        const uint64_t t0 = globaltimer_ns();
-                        while (!mbar_try_wait(smem_u32(&full_bar[s]), issued_parity[s]) &&
-                               globaltimer_ns() - t0 < kWaitLimitNs) {
-                        }
-                    }
-            }
-        } else if (warp == 1 && lane == 0) {
-            // -------------------------------------------------------------- MMA issuer
+        } else if (warp == 1 && lane == 0 && leader) {
+            // -------------------------------------------------------------- MMA issuer (the even CTA of a pair)
             int stage = 0;
             uint32_t phase = 0;
             uint32_t pass_count = 0;   // over all units: selects the accumulator buffer
             bool ok = true;
             Item it;
-            for (int i = 0; ok && get_item(p, i, it); ++i) {
+            for (int i = 0; ok && get_item<kPair>(p, i, it); ++i) {
                 const int passes = 1 + it.h1 - it.h0;
                 for (int pass = 0; ok && pass < passes; ++pass, ++pass_count) {
                     const uint32_t buf = pass_count & 1u;
                     const uint32_t use = (pass_count >> 1) & 1u;
-                    if (!mbar_wait(smem_u32(&acc_empty[buf]), use ^ 1u, abort_flag)) { ok = false; break; }
+                    const bool freed = kPair ? mbar_wait_cluster(smem_u32(&acc_empty[buf]), use ^ 1u, abort_flag)
+                                             : mbar_wait(smem_u32(&acc_empty[buf]), use ^ 1u, abort_flag);
+                    if (!freed) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t d_acc = tmem + buf * kBufCols;
                     for (int kb = 0; kb < p.KB; ++kb) {
-                        if (!mbar_wait(smem_u32(&full_bar[stage]), phase, abort_flag)) { ok = false; break; }
+                        const bool landed = kPair ? mbar_wait_cluster(smem_u32(&full_bar[stage]), phase, abort_flag)
+                                                  : mbar_wait(smem_u32(&full_bar[stage]), phase, abort_flag);
+                        if (!landed) { ok = false; break; }
                         tc_fence_after();
                         const uint32_t st = smem_u32(tiles + stage * kStageBytes);
                         const uint64_t da = smem_desc_k128(st);
-                        const uint64_t dw = smem_desc_k128(st + kTileAct);   // 256 rows: W_gate then W_up
+                        // pair: W_gate here, W_up in the peer; single: W_gate then W_up, 256 rows
+                        const uint64_t dw = smem_desc_k128(st + kTileAct);
 #pragma unroll
                         for (int kk = 0; kk < BK / UK; ++kk) {
                             // advance 16 elements = 32 bytes inside the swizzle atom
                             const uint64_t off = static_cast<uint64_t>((kk * UK * 2) >> 4);
-                            umma_bf16(d_acc, da + off, dw + off, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                            if constexpr (kPair)
+                                umma_bf16_pair(d_acc, da + off, dw + off, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                            else
+                                umma_bf16(d_acc, da + off, dw + off, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
                         }
-                        umma_commit(smem_u32(&empty_bar[stage]));
+                        if constexpr (kPair)
+                            umma_commit_pair(smem_u32(&empty_bar[stage]), 3);
+                        else
+                            umma_commit(smem_u32(&empty_bar[stage]));
                         if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                     }
                     if (!ok) break;
-                    umma_commit(smem_u32(&acc_full[buf]));
+                    if constexpr (kPair)
+                        umma_commit_pair(smem_u32(&acc_full[buf]), 3);
+                    else
+                        umma_commit(smem_u32(&acc_full[buf]));
                 }
             }
-            // Every MMA must have completed before TMEM is released.
-            umma_commit(smem_u32(drain_bar));
-            const uint64_t t0 = globaltimer_ns();
-            while (!mbar_try_wait(smem_u32(drain_bar), 0) && globaltimer_ns() - t0 < kWaitLimitNs) {
-            }
+            // Every MMA must have completed before TMEM or shared memory is released.
+            if constexpr (kPair)
+                umma_commit_pair(smem_u32(drain_bar), 3);
+            else
+                umma_commit(smem_u32(drain_bar));
         }
     } else {
         setmaxnreg_inc<kRegsLarge>();
-        // ------------------------------------------------------------------ epilogue
+        // ------------------------------------------------------------------ epilogue (every CTA)
         const int quad = warp & 3;                         // TMEM lanes 32*quad .. +31 = tokens
         const int half = (warp - kEpiWarp0) >> 2;          // neurons [64*half, 64*half + 64)
         const bool summer = (quad == 0);                   // adds the four quadrants of its half
@@ -291,40 +359,51 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
         uint32_t pass_count = 0, head_count = 0;
         bool ok = true;
         // Adds this warp's two 32-column sums into the four-quadrant sum of its half and, for
-        // the summing warps, writes the 64 results to dst and releases the TMEM buffer.
-        auto reduce_store = [&](const float (&colsum)[2], float* dst, uint32_t buf) -> bool {
+        // the summing warps, writes the 64 results to dst.  Two shared-memory slots are used
+        // alternately; a slot is rewritten only after both summing warps have read it.
+        auto reduce_store = [&](const float (&colsum)[2], float* dst) -> bool {
             const uint32_t slot = head_count & 1u;
-            const uint32_t rphase = (head_count >> 1) & 1u;
+            const uint32_t use = head_count >> 1;
             ++head_count;
             float* rs = red + slot * 4 * BNEU;
-            if (!summer) {
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
-            }
+            if (!mbar_wait(smem_u32(&red_empty[slot]), (use & 1u) ^ 1u, abort_flag)) return false;
             rs[quad * BNEU + half * 64 + lane] = colsum[0];
             rs[quad * BNEU + half * 64 + 32 + lane] = colsum[1];
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&red_full[slot]));
             if (summer) {
                 // the four quadrants of this half, in a fixed order
-                if (!mbar_wait(smem_u32(&red_full[slot]), rphase, abort_flag)) return false;
+                if (!mbar_wait(smem_u32(&red_full[slot]), use & 1u, abort_flag)) return false;
 #pragma unroll
                 for (int b = 0; b < 2; ++b) {
                     const int n = half * 64 + 32 * b + lane;
                     dst[32 * b + lane] = ((rs[n] + rs[BNEU + n]) + rs[2 * BNEU + n]) + rs[3 * BNEU + n];
                 }
-                // only now may the buffer (and, two reductions later, this red slot) be reused
-                tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+                if (lane == 0) mbar_arrive(smem_u32(&red_empty[slot]));
             }
             return true;
         };
+        // Once the pass's last TMEM load has landed in registers the accumulator buffer is free:
+        // release it (in the pair form an arrival on the even CTA's acc_empty) before the math
+        // and the reduction.
+        auto release = [&](uint32_t buf) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                if constexpr (kPair)
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&acc_empty[buf]), 0));
+                else
+                    mbar_arrive(smem_u32(&acc_empty[buf]));
+            }
+        };
         Item it;
-        for (int i = 0; ok && get_item(p, i, it); ++i) {
-            int uc, uj;
-            unit_coords(p, it.unit, uc, uj);
+        for (int i = 0; ok && get_item<kPair>(p, i, it); ++i) {
+            int ucu, uj;
+            unit_coords(p, it.unit, ucu, uj);
+            // chunk uc = TC (the empty half of a last pair) has a slot of its own that the
+            // reduce never reads
+            const int uc = kPair ? 2 * ucu + static_cast<int>(rank) : ucu;
             const int64_t slot_unit = static_cast<int64_t>(uc) * p.NT + uj;   // partial slot: (chunk, tile)
             float* out = p.partial + (slot_unit * p.G + it.h0) * static_cast<int64_t>(BNEU);
             const int passes = 1 + it.h1 - it.h0;
@@ -354,6 +433,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                         tmem_ld16(acc + col_u + 32u * blk, &vu[0]);
                         tmem_ld16(acc + col_u + 32u * blk + 16u, &vu[16]);
                         tmem_wait_ld();
+                        if (blk == 1) release(buf);
 #pragma unroll
                         for (int e = 0; e < 32; ++e) {
                             swiglu_alpha_beta(vg[e], vu[e], alpha[32 * blk + e], beta[32 * blk + e]);
@@ -362,13 +442,8 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                         }
                         asum[blk] = want_act ? butterfly32(vg, lane) : 0.0f;
                     }
-                    if (!want_act) {
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
-                        continue;
-                    }
-                    if (!reduce_store(asum, p.partial_act + slot_unit * BNEU + half * 64, buf)) { ok = false; break; }
+                    if (!want_act) continue;
+                    if (!reduce_store(asum, p.partial_act + slot_unit * BNEU + half * 64)) { ok = false; break; }
                     continue;
                 }
                 // head pass: column sums of Delta^2 over this warp's 32 tokens
@@ -381,6 +456,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                     tmem_ld16(acc + col_u + 32u * blk, &vu[0]);
                     tmem_ld16(acc + col_u + 32u * blk + 16u, &vu[16]);
                     tmem_wait_ld();
+                    if (blk == 1) release(buf);
 #pragma unroll
                     for (int e = 0; e < 32; ++e) {
                         const float dlt = fmaf(alpha[32 * blk + e], d2[e], beta[32 * blk + e] * vu[e]);
@@ -388,16 +464,48 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                     }
                     colsum[blk] = butterfly32(d2, lane);
                 }
-                if (!reduce_store(colsum, out + (pass - 1) * BNEU + half * 64, buf)) { ok = false; break; }
+                if (!reduce_store(colsum, out + (pass - 1) * BNEU + half * 64)) { ok = false; break; }
             }
         }
     }
 
     tc_fence_before();
     __syncthreads();
+    if (warp == 1 && lane == 0) {
+        // the last MMA commit: every MMA (in the pair form reading both CTAs' tiles and writing
+        // both CTAs' TMEM) has completed
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait(smem_u32(drain_bar), 0) && globaltimer_ns() - t0 < kWaitLimitNs) {
+        }
+    }
+    // After a wait gave up, loads already issued (in the pair form also the peer's) may still be
+    // landing in this CTA's shared memory or on its barriers: let them finish before exiting.
+    if constexpr (kPair) {
+        cluster_sync();
+        if (threadIdx.x == 0) {
+            const int peer_abort = static_cast<int>(ld_shared_cluster_u32(
+                mapa_shared(smem_u32(const_cast<int*>(abort_flag)), rank ^ 1u)));
+            if (*abort_flag || peer_abort) {
+                const uint64_t t0 = globaltimer_ns();
+                while (globaltimer_ns() - t0 < 200ull * 1000ull) {
+                }
+            }
+        }
+        cluster_sync();
+    } else {
+        if (threadIdx.x == 0 && *abort_flag) {
+            const uint64_t t0 = globaltimer_ns();
+            while (globaltimer_ns() - t0 < 200ull * 1000ull) {
+            }
+        }
+        __syncthreads();
+    }
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
+        if constexpr (kPair)
+            tmem_dealloc_pair(tmem, kTmemCols);
+        else
+            tmem_dealloc(tmem, kTmemCols);
     }
     if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, static_cast<int>(DTP_ERR_NOT_CONVERGED));
 }
@@ -511,10 +619,16 @@ static bool make_map(CUtensorMap* m, const void* base, int rank, const cuuint64_
     return r == CUDA_SUCCESS;
 }
 
-static size_t partial_bytes(int64_t T, int G, int N) {
+// partial slots: one per (token chunk, neuron tile), for an even number of chunks (the odd
+// CTA of a last, half-empty pair stores into the extra chunk's slots)
+static int64_t slot_units(int64_t T, int N) {
     const int64_t NT = (N + BNEU - 1) / BNEU;
     const int64_t TC = (T + BT - 1) / BT;
-    return static_cast<size_t>(NT * TC) * G * BNEU * sizeof(float);
+    return NT * ((TC + 1) / 2) * 2;
+}
+
+static size_t partial_bytes(int64_t T, int G, int N) {
+    return static_cast<size_t>(slot_units(T, N)) * G * BNEU * sizeof(float);
 }
 
 // bytes of the header and the per-unit A partials (the down-edge activation
@@ -525,9 +639,7 @@ size_t workspace_bytes(int64_t T, int d, int G, int N) {
 }
 
 size_t workspace_bytes_with_act(int64_t T, int d, int G, int N) {
-    const int64_t NT = (N + BNEU - 1) / BNEU;
-    const int64_t TC = (T + BT - 1) / BT;
-    return align_up(workspace_bytes(T, d, G, N), 256) + static_cast<size_t>(NT * TC) * BNEU * sizeof(float);
+    return align_up(workspace_bytes(T, d, G, N), 256) + static_cast<size_t>(slot_units(T, N)) * BNEU * sizeof(float);
 }
 
 // The fixed-order reduce of a workspace's unit partials into A (and act2 when the workspace
@@ -587,7 +699,6 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     p.NT = (N + BNEU - 1) / BNEU;
     p.TC = static_cast<int>((T + BT - 1) / BT);
     p.KB = (d + BK - 1) / BK;
-    p.units = static_cast<int64_t>(p.NT) * p.TC;
     p.status = reinterpret_cast<int*>(workspace);
     p.partial = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(workspace) + kWorkspaceHeader);
     p.T = T;
@@ -600,23 +711,58 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     DTP_CUDA_TRY(cudaGetDevice(&dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev));
-    DTP_CUDA_TRY(cudaFuncSetAttribute(affinity_fo_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(kSmemBytes)));
+    // CTA pairs when all weight tiles fit in half of L2 (no chunk grouping needed), single CTAs
+    // otherwise
+    const double tile_bytes = 2.0 * BNEU * d * 2.0;   // W_gate and W_up rows of one neuron tile
+    const bool weights_fit = static_cast<double>(p.NT) * tile_bytes <= l2 / 2.0;
+    const bool pair = weights_fit;
+    auto kernel = pair ? affinity_fo_tc_kernel<true> : affinity_fo_tc_kernel<false>;
+    const size_t smem = pair ? Form<true>::kSmemBytes : Form<false>::kSmemBytes;
+    DTP_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = pair ? 2 : 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = pair ? 1 : 0;
     const int cap = (max_ctas > 0 && max_ctas < sms) ? max_ctas : sms;
-    const int grid = static_cast<int>(p.units < cap ? p.units : cap);
-    // chunk grouping: keep the weight tiles of the units in flight within a third of L2
-    {
-        const double tile_bytes = 2.0 * BNEU * d * 2.0;
-        p.cg = 1;
-        if (static_cast<double>(p.NT) * tile_bytes > l2 / 2.0)
-            while (p.cg < 64 && p.cg < p.TC && (static_cast<double>(grid) / p.cg) * tile_bytes > l2 / 3.0) p.cg *= 2;
+    int workers;
+    if (pair) {
+        p.TU = (p.TC + 1) / 2;
+        // one CTA pair per two SMs (fewer under max_ctas, rounded down to pairs, at least one
+        // pair), and no more pairs than can be resident at once (queried once per device)
+        cfg.gridDim = dim3(static_cast<unsigned>(sms & ~1), 1, 1);
+        static std::atomic<int> resident_cache[64];
+        int resident = dev < 64 ? resident_cache[dev].load(std::memory_order_relaxed) : 0;
+        if (resident <= 0) {
+            DTP_CUDA_TRY(cudaOccupancyMaxActiveClusters(&resident, kernel, &cfg));
+            if (resident <= 0) return DTP_ERR_CUDA;
+            if (dev < 64) resident_cache[dev].store(resident, std::memory_order_relaxed);
+        }
+        workers = cap / 2 < resident ? cap / 2 : resident;
+        if (workers < 1) workers = 1;
+    } else {
+        p.TU = p.TC;
+        workers = cap;
     }
-    p.full_rounds = static_cast<int>(p.units / grid);
-    const int left = static_cast<int>(p.units - static_cast<int64_t>(p.full_rounds) * grid);
-    p.split = left > 0 ? (grid / left < G ? grid / left : G) : 1;
+    p.units = static_cast<int64_t>(p.NT) * p.TU;
+    if (p.units < workers) workers = static_cast<int>(p.units);
+    // chunk grouping: keep the weight tiles of the units in flight within a third of L2
+    p.cg = 1;
+    if (!weights_fit)
+        while (p.cg < 64 && p.cg < p.TU && (static_cast<double>(workers) / p.cg) * tile_bytes > l2 / 3.0) p.cg *= 2;
+    p.full_rounds = static_cast<int>(p.units / workers);
+    const int left = static_cast<int>(p.units - static_cast<int64_t>(p.full_rounds) * workers);
+    p.split = left > 0 ? (workers / left < G ? workers / left : G) : 1;
     if (p.split < 1) p.split = 1;
     p.tail_items = left * p.split;
-    affinity_fo_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(m_wg, m_wu, m_x, m_c, p);
+    cfg.gridDim = dim3(static_cast<unsigned>(pair ? 2 * workers : workers), 1, 1);
+    DTP_CUDA_TRY(cudaLaunchKernelEx(&cfg, kernel, m_wg, m_wu, m_x, m_c, p));
     DTP_CUDA_TRY(cudaGetLastError());
     if (defer_reduce) return DTP_OK;
     return launch_reduce(workspace, T, d, G, N, A, p.rms ? act2 : nullptr, qpg, stream, 0, 0);

@@ -161,6 +161,34 @@ def test_full_size_sampled_neurons(name):
     assert torch.isfinite(A).all() and (A >= 0).all()
 
 
+@pytest.mark.parametrize("T", [1, 129, 257, 640])
+def test_odd_and_even_token_chunk_counts(T):
+    """Chunk counts 1, 2, 3 and 5: with CTA pairs the odd CTA of a last, half-empty pair reloads
+    the last chunk and its sums go to a spare slot that must not reach A."""
+    d, G, N = 256, 4, 200
+    L = synth.make_layer(d, G, N, T, seed=40 + T, dtype="bf16")
+    A = _gpu(L).cpu().numpy()
+    assert _rel_fro(A, _oracle(L)) <= BF16_TOL
+
+
+@pytest.mark.parametrize("T,max_ctas", [(300, 0), (300, 5), (1000, 151)])
+def test_weights_beyond_half_of_l2(T, max_ctas):
+    """W_gate + W_up of 128 MiB (d = 4096, N = 8192) exceed half of L2, so the kernel runs as
+    single CTAs with chunk grouping; sampled neuron columns against the oracle, and the grid cap
+    leaves A bitwise unchanged."""
+    d, G, N = 4096, 2, 8192
+    L = synth.make_layer(d, G, N, T, seed=60, dtype="bf16")
+    g = {k: v.to(DEV) for k, v in L.items()}
+    A = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"], max_ctas=max_ctas)
+    A_full = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"])
+    torch.cuda.synchronize()
+    assert torch.equal(A, A_full)
+    cols = np.unique(np.concatenate([np.random.default_rng(2).choice(N, size=5, replace=False), [0, 127, 128, N - 1]]))
+    ref = _oracle(L, rows=cols)
+    got = A[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
+    assert _rel_fro(got, ref) <= BF16_TOL
+
+
 @pytest.mark.parametrize("max_ctas", [1, 7, 151])
 def test_grid_cap_does_not_change_the_result(max_ctas):
     """The persistent grid may be capped (SMs left to a concurrent search); A is bitwise the same."""

@@ -34,7 +34,7 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls():
 
 
 def test_noalloc_rejects_calls_beyond_its_scratch():
-    # ceil(T/128) * ceil(N/128) * H_kv = 129 * 16 * 16 > 32768, the documented limit
+    # 129 chunks, rounded up to 130: 130 * ceil(N/128) * H_kv = 130 * 16 * 16 > 32768, the documented limit
     G, N, T, d = 16, 2048, 129 * 128, 8
     X = torch.zeros((T, d), dtype=torch.bfloat16, device=DEV)
     C = torch.zeros((G, T, d), dtype=torch.bfloat16, device=DEV)
