@@ -73,6 +73,28 @@ struct Shared {
 
 __device__ __forceinline__ size_t align_up_dev(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// f(i, a[i]) for every i < n, the block's threads taking consecutive elements: 16-byte loads of
+// four elements when a is 16-byte aligned (the tail, and unaligned arrays, element by element).
+// Every caller's result is independent of the visiting order (a max, an exact integer sum, or an
+// element-wise copy).
+template <class F>
+__device__ __forceinline__ void for_each_a(const float* __restrict__ a, int64_t n, F&& f) {
+    int64_t head = 0;
+    if ((reinterpret_cast<uintptr_t>(a) & 15u) == 0) {
+        const int64_t n4 = n >> 2;
+        const float4* a4 = reinterpret_cast<const float4*>(a);
+        for (int64_t i = threadIdx.x; i < n4; i += kThreads) {
+            const float4 v = a4[i];
+            f(4 * i, v.x);
+            f(4 * i + 1, v.y);
+            f(4 * i + 2, v.z);
+            f(4 * i + 3, v.w);
+        }
+        head = n4 << 2;
+    }
+    for (int64_t i = head + threadIdx.x; i < n; i += kThreads) f(i, a[i]);
+}
+
 // floor(a * 2^(bits-e)) for a finite a >= 0, by shifting the fp32 significand.
 __device__ __forceinline__ int64_t quantize_bits(float a, int e, int bits) {
     const uint32_t b = __float_as_uint(a);
@@ -630,7 +652,7 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
         // A fits beside M and nu: copy it once; every pass then reads shared memory
         float* As = reinterpret_cast<float*>(buf + align_up_dev(static_cast<size_t>(N) * D * sizeof(int64_t) +
                                                                 static_cast<size_t>(N) * sizeof(int32_t), 16));
-        for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) As[i] = A_glob[i];
+        for_each_a(A_glob, static_cast<int64_t>(G) * N, [&](int64_t i, float a) { As[i] = a; });
         __syncthreads();
         L.A = As;
     }
@@ -642,11 +664,10 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     // validity and the fixed-point exponent
     uint32_t amax_bits = 0;
     int bad = 0;
-    for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) {
-        const float a = L.A[i];
+    for_each_a(L.A, static_cast<int64_t>(G) * N, [&](int64_t, float a) {
         if (!(a >= 0.0f) || isinf(a)) bad = 1;
         else amax_bits = max(amax_bits, __float_as_uint(a));
-    }
+    });
     bad = __syncthreads_or(bad);
     const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
     if (bad) {
@@ -661,7 +682,7 @@ search_kernel(const float* __restrict__ A_all, int G, int N, int D, int iters, i
     if (amax > 0.0f) frexpf(amax, &e);
     L.e = e;
     int64_t part = 0;
-    for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) part += quantize(L.A[i], e);
+    for_each_a(L.A, static_cast<int64_t>(G) * N, [&](int64_t, float a) { part += quantize(a, e); });
     const int64_t total = block_sum_i64(part, sh);
     if (threadIdx.x < G) sh.h[threadIdx.x] = (threadIdx.x * D) / G;
     if (threadIdx.x == 0) sh.Jprev = -1;
@@ -768,11 +789,10 @@ __device__ bool layer_prologue(Layer& L, Shared& sh, int64_t* total_out) {
     const int64_t GN = static_cast<int64_t>(L.G) * L.N;
     uint32_t amax_bits = 0;
     int bad = 0;
-    for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
-        const float a = L.A[i];
+    for_each_a(L.A, GN, [&](int64_t, float a) {
         if (!(a >= 0.0f) || isinf(a)) bad = 1;
         else amax_bits = max(amax_bits, __float_as_uint(a));
-    }
+    });
     bad = __syncthreads_or(bad);
     const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
     if (bad) return false;
@@ -782,7 +802,7 @@ __device__ bool layer_prologue(Layer& L, Shared& sh, int64_t* total_out) {
     L.e = e;
     if (total_out) {
         int64_t part = 0;
-        for (int64_t i = threadIdx.x; i < GN; i += kThreads) part += quantize(L.A[i], e);
+        for_each_a(L.A, GN, [&](int64_t, float a) { part += quantize(a, e); });
         *total_out = block_sum_i64(part, sh);
     }
     return true;
@@ -801,7 +821,7 @@ __device__ void layer_view(Layer& L, const float* A_glob, int G, int N, int D, u
     if (use_smem == 2) {
         float* As = reinterpret_cast<float*>(buf + align_up_dev(static_cast<size_t>(N) * D * sizeof(int64_t) +
                                                                 static_cast<size_t>(N) * sizeof(int32_t), 16));
-        for (int64_t i = threadIdx.x; i < static_cast<int64_t>(G) * N; i += kThreads) As[i] = A_glob[i];
+        for_each_a(A_glob, static_cast<int64_t>(G) * N, [&](int64_t i, float a) { As[i] = a; });
         __syncthreads();
         L.A = As;
     }
@@ -989,11 +1009,10 @@ chain_normalize_kernel(const float* __restrict__ S_up, const float* __restrict__
             nu[static_cast<int64_t>(m) * N + k] = static_cast<int>((static_cast<int64_t>(k) * D) / N);
     uint32_t amax_bits = 0;
     int bad = 0;
-    for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
-        const float a = src[i];
+    for_each_a(src, GN, [&](int64_t, float a) {
         if (!(a >= 0.0f) || isinf(a)) bad = 1;
         else amax_bits = max(amax_bits, __float_as_uint(a));
-    }
+    });
     bad = __syncthreads_or(bad);
     const int64_t amax_all = block_max_i64(static_cast<int64_t>(amax_bits), sh);
     if (bad) {
@@ -1007,12 +1026,12 @@ chain_normalize_kernel(const float* __restrict__ S_up, const float* __restrict__
     int e = 0;
     if (amax > 0.0f) frexpf(amax, &e);
     int64_t part = 0;
-    for (int64_t i = threadIdx.x; i < GN; i += kThreads) part += quantize_bits(src[i], e, kNormPreBits);
+    for_each_a(src, GN, [&](int64_t, float a) { part += quantize_bits(a, e, kNormPreBits); });
     const uint64_t total = static_cast<uint64_t>(block_sum_i64(part, sh));
-    for (int64_t i = threadIdx.x; i < GN; i += kThreads) {
-        const uint64_t q = static_cast<uint64_t>(quantize_bits(src[i], e, kNormPreBits));
+    for_each_a(src, GN, [&](int64_t i, float a) {
+        const uint64_t q = static_cast<uint64_t>(quantize_bits(a, e, kNormPreBits));
         dst[i] = total ? static_cast<int64_t>((static_cast<unsigned __int128>(q) << kNormBits) / total) : 0;
-    }
+    });
 }
 
 // M[k,l] = up mass of k from heads of layer i on l + down mass of k into heads of layer i+1 on l;
