@@ -96,12 +96,16 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kBufCols = 256;
 constexpr size_t kRedBytes = 2 * 4 * BNEU * sizeof(float);   // [slot][quadrant][neuron]
 
-// Per form: a stage holds this CTA's activation tile and its weight rows (half of B in the pair
-// form, both halves in the single form); both forms keep 192 KB of stages in flight.
+// Per form: a stage holds kBoxes 64-wide k blocks, each this CTA's activation box and its weight
+// box(es) (half of B in the pair form, both halves in the single form); both forms keep 192 KB of
+// stages in flight.  The pair form takes 128 k columns per stage: its MMA thread then waits on a
+// barrier once per eight MMAs instead of four, which measured ~7% faster than six 64-wide stages.
 template <bool kPair>
 struct Form {
-    static constexpr int STAGES = kPair ? 6 : 4;
-    static constexpr uint32_t kStageBytes = kTileAct + (kPair ? 1u : 2u) * kTileW;
+    static constexpr int kBoxes = kPair ? 2 : 1;
+    static constexpr uint32_t kBoxBytes = kTileAct + (kPair ? 1u : 2u) * kTileW;
+    static constexpr int STAGES = kPair ? 3 : 4;
+    static constexpr uint32_t kStageBytes = kBoxes * kBoxBytes;
     static constexpr uint32_t kIdesc = idesc_bf16_f32(kPair ? 2 * BT : BT, 2 * BNEU);
     static constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + kRedBytes + 256;
 };
@@ -113,6 +117,7 @@ struct Params {
     int TC;           // token chunks
     int TU;           // chunk units: chunk pairs ceil(TC / 2) (pair form) or chunks (single form)
     int KB;           // k blocks of 64 over d
+    int KS;           // stages per pass, ceil(KB / kBoxes)
     int64_t units;    // NT * TU
     int full_rounds;  // rounds in which every worker (CTA pair or CTA) takes one whole unit
     int split;        // head groups per left-over unit
@@ -189,6 +194,8 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                       const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_c,
                       const Params p) {
     constexpr int STAGES = Form<kPair>::STAGES;
+    constexpr int kBoxes = Form<kPair>::kBoxes;
+    constexpr uint32_t kBoxBytes = Form<kPair>::kBoxBytes;
     constexpr uint32_t kStageBytes = Form<kPair>::kStageBytes;
     constexpr uint32_t kIdesc = Form<kPair>::kIdesc;
     extern __shared__ uint8_t smem_raw[];
@@ -267,26 +274,45 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                 const int c = c_raw < p.TC ? c_raw : p.TC - 1;
                 const int passes = 1 + it.h1 - it.h0;
                 for (int pass = 0; ok && pass < passes; ++pass) {
-                    for (int kb = 0; kb < p.KB; ++kb) {
+                    for (int ks = 0; ks < p.KS; ++ks) {
                         if (!mbar_wait(smem_u32(&empty_bar[stage]), phase ^ 1u, abort_flag)) { ok = false; break; }
-                        uint8_t* st = tiles + stage * kStageBytes;
-                        if constexpr (kPair) {
-                            const uint32_t fb = full_lead + static_cast<uint32_t>(stage) * 8u;
-                            if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[stage]), 2 * kStageBytes);
-                            if (pass == 0)
-                                tma_load_2d_pair(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
-                            else
-                                tma_load_3d_pair(smem_u32(st), &tm_c, fb, kb * BK, c * BT, it.h0 + pass - 1);
-                            tma_load_2d_pair(smem_u32(st + kTileAct), leader ? &tm_wg : &tm_wu, fb, kb * BK, j * BNEU);
+                        // k blocks in this stage: kBoxes, fewer in a pass's last stage when KB is odd
+                        const int nb = kBoxes == 1 ? 1 : (p.KB - ks * kBoxes < kBoxes ? p.KB - ks * kBoxes : kBoxes);
+                        const uint32_t st = smem_u32(tiles + stage * kStageBytes);
+                        // loads of k block x0 / BK into box hb of the stage
+                        auto load_box = [&](int hb, uint32_t fb, int x) {
+                            const uint32_t sb = st + hb * kBoxBytes;
+                            if constexpr (kPair) {
+                                if (pass == 0)
+                                    tma_load_2d_pair(sb, &tm_x, fb, x, c * BT);
+                                else
+                                    tma_load_3d_pair(sb, &tm_c, fb, x, c * BT, it.h0 + pass - 1);
+                                tma_load_2d_pair(sb + kTileAct, leader ? &tm_wg : &tm_wu, fb, x, j * BNEU);
+                            } else {
+                                if (pass == 0)
+                                    tma_load_2d(sb, &tm_x, fb, x, c * BT);
+                                else
+                                    tma_load_3d(sb, &tm_c, fb, x, c * BT, it.h0 + pass - 1);
+                                tma_load_2d(sb + kTileAct, &tm_wg, fb, x, j * BNEU);
+                                tma_load_2d(sb + kTileAct + kTileW, &tm_wu, fb, x, j * BNEU);
+                            }
+                        };
+                        const uint32_t fb = kPair ? full_lead + static_cast<uint32_t>(stage) * 8u
+                                                  : smem_u32(&full_bar[stage]);
+                        if constexpr (kBoxes == 1) {
+                            // one k block per stage (the single form): the plain sequence
+                            if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[stage]), (kPair ? 2u : 1u) * kStageBytes);
+                            load_box(0, fb, ks * BK);
                         } else {
-                            const uint32_t fb = smem_u32(&full_bar[stage]);
-                            mbar_arrive_expect_tx(fb, kStageBytes);
-                            if (pass == 0)
-                                tma_load_2d(smem_u32(st), &tm_x, fb, kb * BK, c * BT);
-                            else
-                                tma_load_3d(smem_u32(st), &tm_c, fb, kb * BK, c * BT, it.h0 + pass - 1);
-                            tma_load_2d(smem_u32(st + kTileAct), &tm_wg, fb, kb * BK, j * BNEU);
-                            tma_load_2d(smem_u32(st + kTileAct + kTileW), &tm_wu, fb, kb * BK, j * BNEU);
+                            if (leader)
+                                mbar_arrive_expect_tx(smem_u32(&full_bar[stage]),
+                                                      (kPair ? 2u : 1u) * static_cast<uint32_t>(nb) * kBoxBytes);
+                            if (nb == kBoxes) {
+#pragma unroll
+                                for (int hb = 0; hb < kBoxes; ++hb) load_box(hb, fb, (ks * kBoxes + hb) * BK);
+                            } else {
+                                for (int hb = 0; hb < nb; ++hb) load_box(hb, fb, (ks * kBoxes + hb) * BK);
+                            }
                         }
                         if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                     }
@@ -309,23 +335,38 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                     if (!freed) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t d_acc = tmem + buf * kBufCols;
-                    for (int kb = 0; kb < p.KB; ++kb) {
+                    for (int ks = 0; ks < p.KS; ++ks) {
                         const bool landed = kPair ? mbar_wait_cluster(smem_u32(&full_bar[stage]), phase, abort_flag)
                                                   : mbar_wait(smem_u32(&full_bar[stage]), phase, abort_flag);
                         if (!landed) { ok = false; break; }
                         tc_fence_after();
                         const uint32_t st = smem_u32(tiles + stage * kStageBytes);
-                        const uint64_t da = smem_desc_k128(st);
-                        // pair: W_gate here, W_up in the peer; single: W_gate then W_up, 256 rows
-                        const uint64_t dw = smem_desc_k128(st + kTileAct);
+                        // the four 16-wide K steps of box hb; the first MMA of a pass overwrites
+                        auto mma_box = [&](int hb, bool first) {
+                            const uint64_t da = smem_desc_k128(st + hb * kBoxBytes);
+                            // pair: W_gate here, W_up in the peer; single: W_gate then W_up, 256 rows
+                            const uint64_t dw = smem_desc_k128(st + hb * kBoxBytes + kTileAct);
 #pragma unroll
-                        for (int kk = 0; kk < BK / UK; ++kk) {
-                            // advance 16 elements = 32 bytes inside the swizzle atom
-                            const uint64_t off = static_cast<uint64_t>((kk * UK * 2) >> 4);
-                            if constexpr (kPair)
-                                umma_bf16_pair(d_acc, da + off, dw + off, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
-                            else
-                                umma_bf16(d_acc, da + off, dw + off, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                            for (int kk = 0; kk < BK / UK; ++kk) {
+                                // advance 16 elements = 32 bytes inside the swizzle atom
+                                const uint64_t off = static_cast<uint64_t>((kk * UK * 2) >> 4);
+                                const uint32_t accumulate = (first && kk == 0) ? 0u : 1u;
+                                if constexpr (kPair)
+                                    umma_bf16_pair(d_acc, da + off, dw + off, kIdesc, accumulate);
+                                else
+                                    umma_bf16(d_acc, da + off, dw + off, kIdesc, accumulate);
+                            }
+                        };
+                        if constexpr (kBoxes == 1) {
+                            mma_box(0, ks == 0);
+                        } else {
+                            const int nb = p.KB - ks * kBoxes < kBoxes ? p.KB - ks * kBoxes : kBoxes;
+                            if (nb == kBoxes) {
+#pragma unroll
+                                for (int hb = 0; hb < kBoxes; ++hb) mma_box(hb, ks == 0 && hb == 0);
+                            } else {
+                                for (int hb = 0; hb < nb; ++hb) mma_box(hb, ks == 0 && hb == 0);
+                            }
                         }
                         if constexpr (kPair)
                             umma_commit_pair(smem_u32(&empty_bar[stage]), 3);
@@ -732,6 +773,8 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     cfg.numAttrs = pair ? 1 : 0;
     const int cap = (max_ctas > 0 && max_ctas < sms) ? max_ctas : sms;
     int workers;
+    p.KS = pair ? (p.KB + Form<true>::kBoxes - 1) / Form<true>::kBoxes
+                : (p.KB + Form<false>::kBoxes - 1) / Form<false>::kBoxes;
     if (pair) {
         p.TU = (p.TC + 1) / 2;
         // one CTA pair per two SMs (fewer under max_ctas, rounded down to pairs, at least one
