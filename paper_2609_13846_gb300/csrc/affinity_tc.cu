@@ -753,23 +753,44 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev));
     // CTA pairs when all weight tiles fit in half of L2 (no chunk grouping needed), single CTAs
-    // otherwise
+    // otherwise (and wherever no cluster of two can be resident)
     const double tile_bytes = 2.0 * BNEU * d * 2.0;   // W_gate and W_up rows of one neuron tile
     const bool weights_fit = static_cast<double>(p.NT) * tile_bytes <= l2 / 2.0;
-    const bool pair = weights_fit;
-    auto kernel = pair ? affinity_fo_tc_kernel<true> : affinity_fo_tc_kernel<false>;
-    const size_t smem = pair ? Form<true>::kSmemBytes : Form<false>::kSmemBytes;
-    DTP_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = pair ? 2 : 1;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cfg.attrs = attr;
+    // CTA pairs resident at once, queried once per device (0: not yet; -1: none can be, for
+    // instance on a partition too small for a cluster of two, and the single form runs instead)
+    int resident = 0;
+    if (weights_fit) {
+        static std::atomic<int> resident_cache[64];
+        resident = dev < 64 ? resident_cache[dev].load(std::memory_order_relaxed) : 0;
+        if (resident == 0) {
+            DTP_CUDA_TRY(cudaFuncSetAttribute(affinity_fo_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              static_cast<int>(Form<true>::kSmemBytes)));
+            cfg.gridDim = dim3(static_cast<unsigned>(sms & ~1), 1, 1);
+            cfg.dynamicSmemBytes = Form<true>::kSmemBytes;
+            cfg.numAttrs = 1;
+            if (cudaOccupancyMaxActiveClusters(&resident, affinity_fo_tc_kernel<true>, &cfg) != cudaSuccess ||
+                resident < 1) {
+                (void)cudaGetLastError();
+                resident = -1;
+            }
+            if (dev < 64) resident_cache[dev].store(resident, std::memory_order_relaxed);
+        }
+    }
+    const bool pair = resident > 0;
+    auto kernel = pair ? affinity_fo_tc_kernel<true> : affinity_fo_tc_kernel<false>;
+    const size_t smem = pair ? Form<true>::kSmemBytes : Form<false>::kSmemBytes;
+    DTP_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
+    attr[0].val.clusterDim.x = pair ? 2 : 1;
+    cfg.dynamicSmemBytes = smem;
     cfg.numAttrs = pair ? 1 : 0;
     const int cap = (max_ctas > 0 && max_ctas < sms) ? max_ctas : sms;
     int workers;
@@ -778,15 +799,7 @@ int launch_grouped(const void* X, const void* C, const void* Wg, const void* Wu,
     if (pair) {
         p.TU = (p.TC + 1) / 2;
         // one CTA pair per two SMs (fewer under max_ctas, rounded down to pairs, at least one
-        // pair), and no more pairs than can be resident at once (queried once per device)
-        cfg.gridDim = dim3(static_cast<unsigned>(sms & ~1), 1, 1);
-        static std::atomic<int> resident_cache[64];
-        int resident = dev < 64 ? resident_cache[dev].load(std::memory_order_relaxed) : 0;
-        if (resident <= 0) {
-            DTP_CUDA_TRY(cudaOccupancyMaxActiveClusters(&resident, kernel, &cfg));
-            if (resident <= 0) return DTP_ERR_CUDA;
-            if (dev < 64) resident_cache[dev].store(resident, std::memory_order_relaxed);
-        }
+        // pair), and no more pairs than can be resident at once
         workers = cap / 2 < resident ? cap / 2 : resident;
         if (workers < 1) workers = 1;
     } else {

@@ -466,7 +466,7 @@ static bool map_bf16(CUtensorMap* m, const void* base, int rank, const cuuint64_
 }
 
 // Fills the form-dependent fields of p (row_units, KS, units), launches the main kernel (CTA pairs
-// when B, b_bytes in all, fits in half of L2) and the reduce.  mb0p / mb1p are B's maps for the pair
+// when B, b_bytes in all, fits in half of L2 and a cluster of two can be resident) and the reduce.  mb0p / mb1p are B's maps for the pair
 // form (boxes of 128 rows), mb0 / mb1 for the single form.
 template <int MODE>
 static int run(const CUtensorMap& ma, const CUtensorMap& mb0, const CUtensorMap& mb1, const CUtensorMap& mb0p,
@@ -476,33 +476,46 @@ static int run(const CUtensorMap& ma, const CUtensorMap& mb0, const CUtensorMap&
     DTP_CUDA_TRY(cudaGetDevice(&dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     DTP_CUDA_TRY(cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev));
-    const bool pair = b_bytes <= l2 / 2.0;
-    auto kernel = pair ? sumsq_tc_kernel<MODE, true> : sumsq_tc_kernel<MODE, false>;
-    const size_t smem = pair ? Form<true>::kSmemBytes : Form<false>::kSmemBytes;
-    DTP_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = pair ? 2 : 1;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cfg.attrs = attr;
+    // CTA pairs resident at once, queried once per device and mode (0: not yet; -1: none can be,
+    // and the single form runs instead)
+    int resident = 0;
+    if (b_bytes <= l2 / 2.0) {
+        static std::atomic<int> resident_cache[2][64];
+        resident = dev < 64 ? resident_cache[MODE][dev].load(std::memory_order_relaxed) : 0;
+        if (resident == 0) {
+            DTP_CUDA_TRY(cudaFuncSetAttribute(sumsq_tc_kernel<MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              static_cast<int>(Form<true>::kSmemBytes)));
+            cfg.gridDim = dim3(static_cast<unsigned>(sms & ~1), 1, 1);
+            cfg.dynamicSmemBytes = Form<true>::kSmemBytes;
+            cfg.numAttrs = 1;
+            if (cudaOccupancyMaxActiveClusters(&resident, sumsq_tc_kernel<MODE, true>, &cfg) != cudaSuccess ||
+                resident < 1) {
+                (void)cudaGetLastError();
+                resident = -1;
+            }
+            if (dev < 64) resident_cache[MODE][dev].store(resident, std::memory_order_relaxed);
+        }
+    }
+    const bool pair = resident > 0;
+    auto kernel = pair ? sumsq_tc_kernel<MODE, true> : sumsq_tc_kernel<MODE, false>;
+    const size_t smem = pair ? Form<true>::kSmemBytes : Form<false>::kSmemBytes;
+    DTP_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
+    attr[0].val.clusterDim.x = pair ? 2 : 1;
+    cfg.dynamicSmemBytes = smem;
     cfg.numAttrs = pair ? 1 : 0;
     int workers;
     if (pair) {
         p.row_units = (p.row_chunks + 1) / 2;
         p.KS = (p.KB + Form<true>::kBoxes - 1) / Form<true>::kBoxes;
-        cfg.gridDim = dim3(static_cast<unsigned>(sms & ~1), 1, 1);
-        static std::atomic<int> resident_cache[2][64];
-        int resident = dev < 64 ? resident_cache[MODE][dev].load(std::memory_order_relaxed) : 0;
-        if (resident <= 0) {
-            DTP_CUDA_TRY(cudaOccupancyMaxActiveClusters(&resident, kernel, &cfg));
-            if (resident <= 0) return DTP_ERR_CUDA;
-            if (dev < 64) resident_cache[MODE][dev].store(resident, std::memory_order_relaxed);
-        }
         workers = sms / 2 < resident ? sms / 2 : resident;
     } else {
         p.row_units = p.row_chunks;
