@@ -170,24 +170,6 @@ __device__ __forceinline__ bool get_item(const Params& p, int i, Item& it) {
     return false;
 }
 
-// Sum over the warp's 32 lanes of 32 per-lane columns: afterwards lane L holds
-// the sum of column L.  Each of the 5 rounds halves the columns a lane keeps.
-__device__ __forceinline__ float butterfly32(float (&v)[32], int lane) {
-#pragma unroll
-    for (int r = 0; r < 5; ++r) {
-        const int o = 16 >> r;
-        const int m = 16 >> r;
-        const bool upper = (lane & o) != 0;
-#pragma unroll
-        for (int i = 0; i < m; ++i) {
-            const float send = upper ? v[i] : v[i + m];
-            const float keep = upper ? v[i + m] : v[i];
-            v[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
-        }
-    }
-    return v[0];
-}
-
 template <bool kPair>
 __global__ void __launch_bounds__(kThreads, 1)
 affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_constant__ CUtensorMap tm_wu,
@@ -396,20 +378,45 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
         const uint32_t col_g = static_cast<uint32_t>(half * 64);          // gate columns of this half
         const uint32_t col_u = static_cast<uint32_t>(BNEU + half * 64);   // up columns of this half
+        // The warp reads its 32 lanes (tokens) x 64 neurons as four chunks (h, cb): 16-lane half h,
+        // 32-column block cb, one 16-lane load each of the gate and the up columns.  Register j =
+        // 4 r + q of a chunk is (token 16 h + t/4 + 8 (q >> 1), neuron 32 cb + 8 r + 2 (t % 4) +
+        // (q & 1)) for thread t, so a thread owns 4 tokens x 16 neurons; alpha and beta of its 64
+        // pairs stay in registers for the whole unit, indexed [16 (2 h + cb) + j].
         float alpha[64], beta[64];
         uint32_t pass_count = 0, head_count = 0;
         bool ok = true;
-        // Adds this warp's two 32-column sums into the four-quadrant sum of its half and, for
-        // the summing warps, writes the 64 results to dst.  Two shared-memory slots are used
-        // alternately; a slot is rewritten only after both summing warps have read it.
-        auto reduce_store = [&](const float (&colsum)[2], float* dst) -> bool {
+        // sums over the thread's 4 tokens, per neuron: slot 8 cb + 2 r + (q & 1)
+        auto acc_slot = [](int cb, int j) { return 8 * cb + 2 * (j >> 2) + (j & 1); };
+        // Sums over the 8 lanes that share a thread's neurons (lanes differing in bits 2-4), in a
+        // fixed order: afterwards v[0], v[1] hold neurons n(t), n(t) + 1 of the warp's 64,
+        // n(t) = 32 ((t >> 4) & 1) + 8 ((t >> 2) & 3) + 2 (t & 3).
+        auto butterfly8 = [&](float (&v)[16]) {
+#pragma unroll
+            for (int rd = 0; rd < 3; ++rd) {
+                const int o = 16 >> rd;
+                const int m = 8 >> rd;
+                const bool upper = (lane & o) != 0;
+#pragma unroll
+                for (int i = 0; i < m; ++i) {
+                    const float send = upper ? v[i] : v[i + m];
+                    const float keep = upper ? v[i + m] : v[i];
+                    v[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
+                }
+            }
+        };
+        const int n_t = 32 * ((lane >> 4) & 1) + 8 * ((lane >> 2) & 3) + 2 * (lane & 3);
+        // Adds this warp's 32-token sums (neurons n(t), n(t) + 1 in each thread) into the
+        // four-quadrant sum of its half and, for the summing warps, writes the 64 results to dst.
+        // Two shared-memory slots are used alternately; a slot is rewritten only after both
+        // summing warps have read it.
+        auto reduce_store = [&](float s0, float s1, float* dst) -> bool {
             const uint32_t slot = head_count & 1u;
             const uint32_t use = head_count >> 1;
             ++head_count;
             float* rs = red + slot * 4 * BNEU;
             if (!mbar_wait(smem_u32(&red_empty[slot]), (use & 1u) ^ 1u, abort_flag)) return false;
-            rs[quad * BNEU + half * 64 + lane] = colsum[0];
-            rs[quad * BNEU + half * 64 + 32 + lane] = colsum[1];
+            *reinterpret_cast<float2*>(rs + quad * BNEU + half * 64 + n_t) = make_float2(s0, s1);
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&red_full[slot]));
             if (summer) {
@@ -454,58 +461,63 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
                 if (!mbar_wait(smem_u32(&acc_full[buf]), use, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t acc = lane_base + buf * kBufCols;
+                float sums[16];
+#pragma unroll
+                for (int k = 0; k < 16; ++k) sums[k] = 0.0f;
                 if (pass == 0) {
                     // operating point; optionally the down-edge activation sums
                     const bool want_act = p.rms != nullptr && it.h0 == 0;
-                    float ir2 = 0.0f;
+                    float ir2[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // tokens 16 h + t/4 + 8 s, slot 2 h + s
                     if (want_act) {
-                        const int64_t tok = static_cast<int64_t>(uc) * BT + quad * 32 + lane;
-                        if (tok < p.T) {
-                            const float r = p.rms[tok];
-                            ir2 = 1.0f / (r * r);
+#pragma unroll
+                        for (int ts = 0; ts < 4; ++ts) {
+                            const int64_t tok = static_cast<int64_t>(uc) * BT + quad * 32 + 16 * (ts >> 1) +
+                                                (lane >> 2) + 8 * (ts & 1);
+                            if (tok < p.T) {
+                                const float r = p.rms[tok];
+                                ir2[ts] = 1.0f / (r * r);
+                            }
                         }
                     }
-                    float asum[2];
 #pragma unroll
-                    for (int blk = 0; blk < 2; ++blk) {
-                        float vg[32], vu[32];
-                        tmem_ld16(acc + col_g + 32u * blk, &vg[0]);
-                        tmem_ld16(acc + col_g + 32u * blk + 16u, &vg[16]);
-                        tmem_ld16(acc + col_u + 32u * blk, &vu[0]);
-                        tmem_ld16(acc + col_u + 32u * blk + 16u, &vu[16]);
+                    for (int ch = 0; ch < 4; ++ch) {
+                        const int h = ch >> 1, cb = ch & 1;
+                        float vg[16], vu[16];
+                        const uint32_t lanes = static_cast<uint32_t>(16 * h) << 16;
+                        tmem_ld_16x256b_x4(acc + lanes + col_g + 32u * cb, vg);
+                        tmem_ld_16x256b_x4(acc + lanes + col_u + 32u * cb, vu);
                         tmem_wait_ld();
-                        if (blk == 1) release(buf);
+                        if (ch == 3) release(buf);
 #pragma unroll
-                        for (int e = 0; e < 32; ++e) {
-                            swiglu_alpha_beta(vg[e], vu[e], alpha[32 * blk + e], beta[32 * blk + e]);
-                            const float act = beta[32 * blk + e] * vu[e];   // silu(g) u
-                            vg[e] = act * act * ir2;
+                        for (int j = 0; j < 16; ++j) {
+                            swiglu_alpha_beta(vg[j], vu[j], alpha[16 * ch + j], beta[16 * ch + j]);
+                            const float act = beta[16 * ch + j] * vu[j];   // silu(g) u
+                            sums[acc_slot(cb, j)] = fmaf(act * act, ir2[2 * h + ((j >> 1) & 1)], sums[acc_slot(cb, j)]);
                         }
-                        asum[blk] = want_act ? butterfly32(vg, lane) : 0.0f;
                     }
                     if (!want_act) continue;
-                    if (!reduce_store(asum, p.partial_act + slot_unit * BNEU + half * 64)) { ok = false; break; }
+                    butterfly8(sums);
+                    if (!reduce_store(sums[0], sums[1], p.partial_act + slot_unit * BNEU + half * 64)) { ok = false; break; }
                     continue;
                 }
-                // head pass: column sums of Delta^2 over this warp's 32 tokens
-                float colsum[2];
+                // head pass: sums of Delta^2 over this warp's 32 tokens
 #pragma unroll
-                for (int blk = 0; blk < 2; ++blk) {
-                    float d2[32], vu[32];
-                    tmem_ld16(acc + col_g + 32u * blk, &d2[0]);
-                    tmem_ld16(acc + col_g + 32u * blk + 16u, &d2[16]);
-                    tmem_ld16(acc + col_u + 32u * blk, &vu[0]);
-                    tmem_ld16(acc + col_u + 32u * blk + 16u, &vu[16]);
+                for (int ch = 0; ch < 4; ++ch) {
+                    const int h = ch >> 1, cb = ch & 1;
+                    float pg[16], pu[16];
+                    const uint32_t lanes = static_cast<uint32_t>(16 * h) << 16;
+                    tmem_ld_16x256b_x4(acc + lanes + col_g + 32u * cb, pg);
+                    tmem_ld_16x256b_x4(acc + lanes + col_u + 32u * cb, pu);
                     tmem_wait_ld();
-                    if (blk == 1) release(buf);
+                    if (ch == 3) release(buf);
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        const float dlt = fmaf(alpha[32 * blk + e], d2[e], beta[32 * blk + e] * vu[e]);
-                        d2[e] = dlt * dlt;
+                    for (int j = 0; j < 16; ++j) {
+                        const float dlt = fmaf(alpha[16 * ch + j], pg[j], beta[16 * ch + j] * pu[j]);
+                        sums[acc_slot(cb, j)] = fmaf(dlt, dlt, sums[acc_slot(cb, j)]);
                     }
-                    colsum[blk] = butterfly32(d2, lane);
                 }
-                if (!reduce_store(colsum, out + (pass - 1) * BNEU + half * 64)) { ok = false; break; }
+                butterfly8(sums);
+                if (!reduce_store(sums[0], sums[1], out + (pass - 1) * BNEU + half * 64)) { ok = false; break; }
             }
         }
     }
