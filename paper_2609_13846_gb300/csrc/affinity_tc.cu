@@ -48,13 +48,15 @@
 // 256 columns used by passes alternately, so the epilogue of one pass
 // overlaps the MMAs of the next.
 //
-// Epilogue.  Thread = one token (its TMEM lane); two warps per lane quadrant
-// split the 128 neurons into halves of 64.  Pass 0 leaves alpha = silu'(g) u
-// and beta = silu(g) of the thread's 64 (token, neuron) pairs in registers for
-// the whole unit.  A head pass forms Delta^2 for the same pairs and sums it
-// over tokens: a shuffle butterfly within the warp (32 tokens), then the four
-// quadrant warps' sums are added in shared memory in a fixed order.  The
-// T x G x N intermediate never leaves the SM; each unit writes its G x 128
+// Epilogue.  Two warps per TMEM lane quadrant (32 tokens) split the 128
+// neurons into halves of 64.  A warp reads its accumulator with 16-lane loads
+// (tcgen05.ld 16x256b), so each thread owns 4 tokens x 16 neurons.  Pass 0
+// leaves alpha = silu'(g) u and beta = silu(g) of the thread's 64 (token,
+// neuron) pairs in registers for the whole unit.  A head pass forms Delta^2 for
+// the same pairs, sums it over the thread's 4 tokens (fused multiply-adds),
+// then over the 8 lanes sharing its neurons (a 3-round shuffle butterfly), and
+// the four quadrant warps' sums are added in shared memory in a fixed order.
+// The T x G x N intermediate never leaves the SM; each unit writes its G x 128
 // partial sums to its own workspace slot and a second kernel adds them into A
 // in a fixed order, so the result is deterministic.
 //
