@@ -174,7 +174,7 @@ def cpu_baseline(w, A_gpu, budget_s: float):
     t0 = time.perf_counter()
     oracle.affinity_fo(X, C, Wg, Wu)
     per_tok = (time.perf_counter() - t0) / T0
-    T_slice = int(max(T0, min(2048, budget_s / max(per_tok, 1e-9))))
+    T_slice = int(max(T0, min(8192, budget_s / max(per_tok, 1e-9))))
     L = synth.make_workload_layer(w, T=T_slice)
     X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
     t0 = time.perf_counter()
