@@ -303,6 +303,23 @@ int dtp_affinity_accumulate_noalloc(const void* X, const void* C, const void* W_
  */
 int dtp_workspace_status(const void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * Self-test of the bounded device-side waits every kernel here relies on (no
+ * paper passage: a check of this library's failure reporting).  One block:
+ * thread 0 waits on an mbarrier with limit_ns (1 us .. 1 s); with complete = 0
+ * nothing ever arrives, the wait gives up, sets the shared abort flag and the
+ * workspace status word (DTP_ERR_NOT_CONVERGED), and a second thread waiting
+ * on another never-completed barrier with the library's own limit (2 s) must
+ * leave on that flag; with complete = 1 another warp arrives first and the
+ * status stays DTP_OK.  Writes the two waits' durations (ns) to
+ * elapsed_ns[0..1] (host, 2 entries; the second is 0 when complete = 1) and
+ * synchronises `stream`.  Read the status with dtp_workspace_status.
+ * workspace: device, at least 256 bytes.  DTP_ERR_ARG for a null pointer, a
+ * small workspace or a limit outside the range.
+ */
+int dtp_selftest_bounded_wait(uint64_t limit_ns, int complete, void* workspace, size_t workspace_bytes,
+                              uint64_t* elapsed_ns, void* stream);
+
 /* ------------------------------------------------------------------------ */
 /* 2. Layout optimiser (Sec. 3 "Objective", "Optimiser")                     */
 /* ------------------------------------------------------------------------ */

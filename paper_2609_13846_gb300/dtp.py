@@ -94,6 +94,7 @@ def lib():
                                    ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp, _vp, _sz, _vp]
     L.dtp_affinity_top_share.argtypes = [_vp, _i32, _i32, _i32, _vp, _vp]
     L.dtp_workspace_status.argtypes = [_vp, _sz, _vp]
+    L.dtp_selftest_bounded_wait.argtypes = [ctypes.c_uint64, _i32, _vp, _sz, ctypes.POINTER(ctypes.c_uint64), _vp]
     L.dtp_search_workspace_size.argtypes = [_i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
     L.dtp_search_layout.argtypes = [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
     L.dtp_search_layout_batched.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
@@ -110,7 +111,7 @@ def lib():
                "dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
                "dtp_affinity_finalize",
                "dtp_down_sqnorm", "dtp_workspace_status", "dtp_search_workspace_size", "dtp_search_layout",
-               "dtp_search_layout_batched"):
+               "dtp_search_layout_batched", "dtp_selftest_bounded_wait"):
         getattr(L, fn).restype = _i32
     _lib = L
     return L
@@ -400,6 +401,17 @@ def affinity_accumulate_noalloc(X: torch.Tensor, C: torch.Tensor, W_gate: torch.
 def workspace_status(workspace: torch.Tensor, stream=None) -> int:
     """Synchronise and read the workspace status word (DTP_OK or DTP_ERR_NOT_CONVERGED)."""
     return int(lib().dtp_workspace_status(_ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def selftest_bounded_wait(limit_ns: int, complete: bool, device="cuda:0", stream=None) -> dict:
+    """Run the bounded-wait self-test: a device wait with limit_ns that is (complete) or is not
+    satisfied.  Returns the workspace status and the two waits' durations in ns."""
+    ws = torch.zeros(256, dtype=torch.uint8, device=device)
+    el = (ctypes.c_uint64 * 2)()
+    _check("dtp_selftest_bounded_wait",
+           lib().dtp_selftest_bounded_wait(int(limit_ns), 1 if complete else 0, _ptr(ws), ws.numel(), el,
+                                           _stream(stream)))
+    return {"status": workspace_status(ws, stream), "elapsed_ns": (int(el[0]), int(el[1]))}
 
 
 def affinity_finalize(A: torch.Tensor, T_total: int, wd_sqnorm: torch.Tensor | None = None, stream=None):

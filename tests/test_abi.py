@@ -188,3 +188,17 @@ def test_apply_layout_argument_checks(lib):
     assert lib.dtp_apply_layout(p, p, 2, 8, 64, 4, 2, 16, 64, 2, ptrs, same, p, p, p, ws, None) == -1
     assert lib.dtp_apply_layout(p, p, 2, 8, 64, 4, 2, 16, 64, 2, None, outs, p, p, p, ws, None) == -1
     assert lib.dtp_apply_layout(p, p, 2, 8, 64, 4, 2, 16, 64, 2, ptrs, outs, p, p, None, ws, None) == -5
+
+
+def test_selftest_bounded_wait_rejects_bad_arguments(lib):
+    """The bounded-wait self-test validates its arguments on the host, before any CUDA call."""
+    import ctypes as ct
+    from paper_2609_13846_gb300 import dtp
+    el = (ct.c_uint64 * 2)()
+    dummy = ct.c_void_p(256)   # never dereferenced: every call below fails validation first
+    assert lib.dtp_selftest_bounded_wait(10 ** 6, 0, None, 256, el, None) == dtp.DTP_ERR_ARG
+    assert lib.dtp_selftest_bounded_wait(10 ** 6, 0, dummy, 64, el, None) == dtp.DTP_ERR_ARG
+    assert lib.dtp_selftest_bounded_wait(10 ** 6, 0, dummy, 256, None, None) == dtp.DTP_ERR_ARG
+    assert lib.dtp_selftest_bounded_wait(10, 0, dummy, 256, el, None) == dtp.DTP_ERR_ARG
+    assert lib.dtp_selftest_bounded_wait(2 * 10 ** 9, 0, dummy, 256, el, None) == dtp.DTP_ERR_ARG
+    assert lib.dtp_selftest_bounded_wait(10 ** 6, 2, dummy, 256, el, None) == dtp.DTP_ERR_ARG
