@@ -153,3 +153,25 @@ def test_chain_score_rejects_out_of_range_layout():
         dtp.chain_score(torch.as_tensor(Su, device=DEV), torch.as_tensor(Sd, device=DEV),
                         torch.as_tensor(h, device=DEV), torch.as_tensor(nu, device=DEV), 4)
     assert e.value.status == dtp.DTP_ERR_ARG
+
+
+@pytest.mark.parametrize("D", [2, 4])
+def test_random_layouts_score_one_over_D_per_edge(D):
+    """A uniform random balanced layout co-locates 1/D of each edge's mass in expectation (Sec. 3: a
+    random layout scores (2L-1)/D): the mean over 256 seeded layouts, each scored on the GPU, lies
+    within five standard errors of 1/D on every edge and of (2L-1)/D in total."""
+    L, G, N = 4, 8, 3072
+    Su, Sd = _model(L, G, N, seed=77)
+    gSu = torch.as_tensor(Su, device=DEV).contiguous()
+    gSd = torch.as_tensor(Sd, device=DEV).contiguous()
+    n = 256
+    edges = []
+    for seed in range(2000, 2000 + n):
+        h, nu = ablation.random_layout(L, G, N, D, seed)
+        r = dtp.chain_score(gSu, gSd, torch.as_tensor(h, device=DEV), torch.as_tensor(nu, device=DEV), D)
+        edges.append(r["edge_q"].double().cpu() / 2.0 ** 43)
+    E = torch.stack(edges)                       # [n, 2L-1] co-located fraction of each edge
+    se = E.std(0) / n ** 0.5
+    assert torch.all((E.mean(0) - 1.0 / D).abs() <= 5 * se + 1e-4), (E.mean(0), se)
+    J = E.sum(1)
+    assert abs(float(J.mean()) - (2 * L - 1) / D) <= 5 * float(J.std()) / n ** 0.5 + 1e-4
