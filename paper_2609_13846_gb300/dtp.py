@@ -34,7 +34,8 @@ _sz = ctypes.c_size_t
 
 
 class AffinityOpts(ctypes.Structure):
-    """dtp_affinity_opts: max_ctas caps the persistent grid (0 = one CTA per SM)."""
+    """dtp_affinity_opts: max_ctas caps the persistent grid (0 = one CTA per SM; rounded down to an
+    even count when the kernel runs as CTA pairs)."""
     _fields_ = [("max_ctas", ctypes.c_int), ("flags", ctypes.c_int), ("reserved", ctypes.c_int * 6)]
 
 
@@ -177,8 +178,9 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
 
     X [T,d], C [H_kv,T,d], W_gate/W_up [N,d]: contiguous CUDA tensors, all bf16
     or all fp32.  ``A`` is accumulated into (a zero tensor is made if None).
-    max_ctas > 0 caps the bf16 kernel's persistent grid (SMs left to other streams); with
-    defer_reduce only the main kernel runs and affinity_reduce(workspace, ...) finishes A later.
+    max_ctas > 0 caps the bf16 kernel's persistent grid (SMs left to other streams; rounded down
+    to an even count, at least 2, when the kernel runs as CTA pairs); with defer_reduce only the
+    main kernel runs and affinity_reduce(workspace, ...) finishes A later.
     """
     for name, t in (("X", X), ("C", C), ("W_gate", W_gate), ("W_up", W_up)):
         if not t.is_cuda or not t.is_contiguous():
