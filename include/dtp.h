@@ -12,7 +12,11 @@
  *   - Tensor arguments are DEVICE pointers owned by the caller; the library
  *     never frees or retains them.  Scratch memory is passed in as a
  *     caller-owned device workspace whose size the *_workspace_size query
- *     returns.  The library allocates no device memory.
+ *     returns.  No call allocates device memory.  The one exception to the
+ *     workspace rule is dtp_affinity_accumulate_noalloc, whose scratch is a
+ *     fixed 16 MiB + 256 B array that the library holds on every GPU that
+ *     loads it (a static device array, reserved when the library's module is
+ *     loaded, not by any call).
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Calls are asynchronous on it unless stated otherwise.
  *   - Arrays are row-major, contiguous, 16-byte aligned.
@@ -278,8 +282,9 @@ int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, voi
  * must not grow after start-up).  The paper has no counterpart: this entry
  * point only changes where the scratch lives.
  *
- * Same arguments, layouts, accumulation and result as dtp_affinity_accumulate
- * (bf16 inputs only), minus the workspace.  Scratch comes from one fixed
+ * Same arguments, layouts and accumulation as dtp_affinity_accumulate (bf16
+ * inputs only), minus the workspace; the same kernels in the same launch
+ * shape give A bit for bit equal to that call's.  Scratch comes from one fixed
  * device array of 16 MiB + 256 B inside the library, present on every GPU
  * that loads it until the process exits; the call allocates nothing.
  *   - Limit: c * ceil(N/128) * H_kv <= 32768 per call, with c = ceil(T/128)
@@ -288,12 +293,30 @@ int dtp_down_sqnorm(const void* W_down, int d, int N, int dtype, float* out, voi
  *   - Every call shares the array and it keeps the last call's contents:
  *     calls that overlap on the GPU race and must be serialised by the caller.
  *   - The first call on a device looks up the array's device address with
- *     that device current; make it before any stream capture begins.
+ *     that device current; make it before any stream capture begins.  The
+ *     address is kept for the life of the process: no call may follow a
+ *     cudaDeviceReset of that device.
+ *   - A bounded device-side wait that gives up leaves the partial sums of
+ *     its units unwritten, and the reduce still adds every slot into A, so A
+ *     is then wrong.  The kernels record this in the array's status word:
+ *     dtp_affinity_noalloc_status reads it back after the call.
  * Asynchronous on `stream`.
  */
 int dtp_affinity_accumulate_noalloc(const void* X, const void* C, const void* W_gate,
                                     const void* W_up, int64_t T, int d, int H_kv, int N, float* A,
                                     void* stream);
+
+/*
+ * Device-side status of the last dtp_affinity_accumulate_noalloc call on the
+ * current device (no paper passage: this library's failure reporting).
+ * Synchronises `stream` (pass the stream of that call), then reads the status
+ * word in the library's fixed scratch array: DTP_OK, or DTP_ERR_NOT_CONVERGED
+ * if a bounded wait of the call's kernels gave up (A is then not valid).
+ * Calls of dtp_affinity_accumulate_noalloc that are still queued on other
+ * streams may overwrite the word; order them before this read.  Returns
+ * DTP_ERR_CUDA if the copy or the synchronisation fails.  Allocates nothing.
+ */
+int dtp_affinity_noalloc_status(void* stream);
 
 /*
  * Synchronises `stream`, then reads the status word that kernels of the last

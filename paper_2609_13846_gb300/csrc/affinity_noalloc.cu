@@ -17,7 +17,11 @@
 // from different host threads without ordering) race on it and must be
 // serialised by the caller.  The first call on a device looks up the array's
 // device address (cudaGetSymbolAddress) with that device current; make that
-// first call before any stream capture begins.
+// first call before any stream capture begins.  The address is kept for the
+// life of the process, so no call may follow a cudaDeviceReset of that device.
+//
+// Device-side failures (a bounded wait that gave up) are recorded in the
+// array's status word, which dtp_affinity_noalloc_status reads back.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -85,4 +89,15 @@ extern "C" int dtp_affinity_accumulate_noalloc(const void* X, const void* C, con
     // The status word must start at zero; the partial sums are all written before they are read.
     if (cudaMemsetAsync(scratch, 0, dtp::kWorkspaceHeader, s) != cudaSuccess) return DTP_ERR_CUDA;
     return dtp::tc::launch(X, C, W_gate, W_up, T, d, H_kv, N, A, scratch, s, nullptr, nullptr);
+}
+
+extern "C" int dtp_affinity_noalloc_status(void* stream) {
+    void* scratch = nullptr;
+    const int rc = scratch_address(&scratch);
+    if (rc != DTP_OK) return rc;
+    int st = 0;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(&st, scratch, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess) return DTP_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return DTP_ERR_CUDA;
+    return st == 0 ? DTP_OK : st;
 }

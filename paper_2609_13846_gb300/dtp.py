@@ -63,6 +63,7 @@ def lib():
     L.dtp_affinity_finalize.argtypes = [_vp, _i32, _i32, _i64, _vp, _vp]
     L.dtp_down_sqnorm.argtypes = [_vp, _i32, _i32, _i32, _vp, _vp]
     L.dtp_affinity_accumulate_noalloc.argtypes = [_vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _vp, _vp]
+    L.dtp_affinity_noalloc_status.argtypes = [_vp]
     L.dtp_affinity_accumulate_ex.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _vp,
                                              _sz, _vp]
     L.dtp_affinity_grouped_workspace_size.argtypes = [_i64, _i32, _i32, _i32, _i32, _i32, ctypes.POINTER(_sz)]
@@ -110,7 +111,7 @@ def lib():
                "dtp_affinity_accumulate_ex", "dtp_affinity_add_workspace_size", "dtp_affinity_add_accumulate",
                "dtp_down_weight_workspace_size", "dtp_down_weight_sqnorm", "dtp_down_finalize",
                "dtp_affinity_workspace_size", "dtp_affinity_accumulate", "dtp_affinity_accumulate_noalloc",
-               "dtp_affinity_finalize",
+               "dtp_affinity_noalloc_status", "dtp_affinity_finalize",
                "dtp_down_sqnorm", "dtp_workspace_status", "dtp_search_workspace_size", "dtp_search_layout",
                "dtp_search_layout_batched", "dtp_selftest_bounded_wait"):
         getattr(L, fn).restype = _i32
@@ -389,7 +390,8 @@ def affinity_accumulate_noalloc(X: torch.Tensor, C: torch.Tensor, W_gate: torch.
 
     For callers that cannot allocate device memory; the caller passes the
     inputs and the fp32 output A [H_kv, N], which is accumulated into.  Calls
-    that overlap on the GPU share the scratch and race.
+    that overlap on the GPU share the scratch and race.  A device-side failure
+    is reported by ``affinity_noalloc_status``, not by this call.
     """
     T, d = X.shape
     H = C.shape[0]
@@ -398,6 +400,12 @@ def affinity_accumulate_noalloc(X: torch.Tensor, C: torch.Tensor, W_gate: torch.
                                                _stream(stream))
     _check("dtp_affinity_accumulate_noalloc", st)
     return A
+
+
+def affinity_noalloc_status(stream=None) -> int:
+    """Synchronise ``stream`` and read the status word of the last allocation-free affinity call
+    on the current device (DTP_OK or DTP_ERR_NOT_CONVERGED)."""
+    return int(lib().dtp_affinity_noalloc_status(_stream(stream)))
 
 
 def workspace_status(workspace: torch.Tensor, stream=None) -> int:
