@@ -33,6 +33,24 @@ def _oracle(L, rows=None):
     return oracle.affinity_fo(X, C, Wg, Wu)
 
 
+def _sample_columns(N, n_random, seed):
+    """Neuron columns for a full-size check: one whole 128-neuron tile in the middle of the grid, the
+    last tile (in chunk-major unit order its units are the left-over ones that may be split by heads),
+    the first column and a few random ones."""
+    mid = (N // 128) // 2 * 128
+    rng = np.random.default_rng(seed)
+    cols = [np.arange(mid, min(mid + 128, N)), np.arange(max(N - 128, 0), N), [0],
+            rng.choice(N, size=n_random, replace=False)]
+    return np.unique(np.concatenate(cols))
+
+
+def _check_columns(got, ref):
+    """Relative Frobenius error over the sampled columns, and every entry within the elementwise
+    bound of the ragged-shape tests."""
+    assert _rel_fro(got, ref) <= BF16_TOL
+    assert np.all(np.abs(got - ref) <= 2e-2 * np.abs(ref) + 1e-6 * np.abs(ref).max())
+
+
 def _gpu(L, A=None):
     g = {k: v.to(DEV) for k, v in L.items()}
     out = dtp.affinity_accumulate(g["X"], g["C"], g["W_gate"], g["W_up"], A=A)
@@ -151,13 +169,12 @@ def test_full_size_sampled_neurons(name):
     A_capped = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"], max_ctas=sms - 1)
     torch.cuda.synchronize()
     assert torch.equal(A, A_capped)
-    rng = np.random.default_rng(0)
-    cols = np.sort(rng.choice(w.N, size=6, replace=False))
-    cols = np.unique(np.concatenate([cols, [0, w.N - 1]]))
+    cols = _sample_columns(w.N, 6, seed=0)
+    assert len(cols) >= 136
     Lh = {k: v.cpu() for k, v in L.items()}
     ref = _oracle(Lh, rows=cols)
-    got = A[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
-    assert _rel_fro(got, ref) <= BF16_TOL
+    got = A_capped[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
+    _check_columns(got, ref)
     assert torch.isfinite(A).all() and (A >= 0).all()
 
 
@@ -210,15 +227,15 @@ def test_full_model_layer_sampled_neurons_with_down_term(name):
     Dn = synth.make_down_inputs(w.d, w.G, w.qkv_rows, w.N, w.T, seed=w.seed + 1000, device=DEV)
     A, act2 = dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"])
     torch.cuda.synchronize()
-    rng = np.random.default_rng(1)
-    cols = np.unique(np.concatenate([rng.choice(w.N, size=3, replace=False), [0, w.N - 1]]))
+    cols = _sample_columns(w.N, 3, seed=1)
+    assert len(cols) >= 136
     Lh = {k: v.cpu() for k, v in L.items()}
     ref = _oracle(Lh, rows=cols)
     got = A[:, torch.as_tensor(cols, device=DEV)].double().cpu().numpy()
-    assert _rel_fro(got, ref) <= BF16_TOL
+    _check_columns(got, ref)
     ref_act = oracle.down_activation(Lh["X"].double().numpy(), Lh["W_gate"][cols].double().numpy(),
                                      Lh["W_up"][cols].double().numpy(), Dn["rms"].double().cpu().numpy())
-    assert _rel_fro(act2[torch.as_tensor(cols, device=DEV)].double().cpu().numpy(), ref_act) <= BF16_TOL
+    _check_columns(act2[torch.as_tensor(cols, device=DEV)].double().cpu().numpy(), ref_act)
 
 
 @pytest.mark.parametrize("with_act", [False, True])

@@ -148,6 +148,48 @@ def test_neuron_step_matches_hungarian(N, D):
             assert sorted(r2c.tolist()) == list(range(N))
 
 
+def _qwen_layer_q(layer, T=64):
+    """Exact scores of a Qwen3-0.6B-shaped layer (G = 8, N = 3072) from the oracle's affinity on a
+    token slice of that layer's synthetic activations."""
+    L = synth.make_workload_layer(synth.WORKLOADS["qwen3_0.6b_model"], layer, T=T)
+    A = oracle.affinity_fo(*(L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up")))
+    q, _ = oracle.quantize(A.astype(np.float32))
+    return q
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("case", ["qwen_layer0", "qwen_layer1", "integer"])
+def test_neuron_step_matches_hungarian_at_qwen_size(case):
+    """Qwen-sized cross-check of the exact balanced assignment (Sec. 3 "Optimiser": a linear
+    assignment on I/L replicated slots): N = 3072 neurons, D = 4, the 3072 x 3072 slot-expanded
+    matrix solved by the textbook Hungarian method (O(n^3), about 20 s each) must reach the same
+    optimum as the oracle's successive-shortest-path solver, for two layers of continuous scores
+    (unique optimum certified) and one tie-heavy integer layer."""
+    N, D = 3072, 4
+    if case == "integer":
+        _, q = _rand_q(8, N, 31, "integer")
+        h = np.array([0, 0, 1, 1, 2, 2, 3, 3], dtype=np.int32)
+    else:
+        layer = int(case[-1])
+        q = _qwen_layer_q(layer)
+        h = np.array([0, 0, 1, 1, 2, 2, 3, 3] if layer == 0 else [0, 1, 2, 3, 3, 2, 1, 0], dtype=np.int32)
+    M = np.zeros((N, D), dtype=np.int64)
+    for g in range(q.shape[0]):
+        M[:, h[g]] += q[g]
+    cap = N // D
+    total, r2c = oracle.hungarian_max(np.repeat(M, cap, axis=1))
+    assert sorted(r2c.tolist()) == list(range(N))
+    assert int(M[np.arange(N), r2c // cap].sum()) == total  # the Hungarian's own assignment
+    nu, uniq = oracle.neuron_step(q, h, D)
+    assert np.bincount(nu, minlength=D).tolist() == [cap] * D
+    assert oracle.assignment_gain(q, h, nu, D) == total
+    if case == "integer":
+        assert not uniq  # integer scores in a small range: many optima, the tie-break decides
+    else:
+        assert uniq
+        np.testing.assert_array_equal(nu, r2c // cap)  # a unique optimum: the same assignment
+
+
 def test_neuron_step_d2_is_a_sort():
     """D = 2 reduces to sorting M_k0 - M_k1 (textbook): device 0 takes the top half."""
     _, q = _rand_q(4, 200, 5)
