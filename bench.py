@@ -49,23 +49,29 @@ def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         j = json.load(open(p))
+        clk = j.get("clocks_under_load", {})
         return dict(bf16=float(j["bf16_tflops"]), bf16_sustained=float(j.get("bf16_tflops_sustained", 0)),
-                    hbm=float(j["hbm_gbs"]), source="measured")
-    return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
+                    hbm=float(j["hbm_gbs"]), source="measured", sm_mhz=clk.get("sm_mhz_median"))
+    return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback", sm_mhz=None)
 
 
-def traffic_from_profile():
-    """DRAM bytes per launch of the affinity kernel from the committed ncu summary, if current."""
-    p = os.path.join(ROOT, "profiles", "affinity_fo_tc_qwen3_layer.txt")
+def profile_field(key: str, name: str = "affinity_fo_tc_qwen3_layer.txt"):
+    """A number from a committed ncu summary under profiles/ (a line ``key: value ...``), or None."""
+    p = os.path.join(ROOT, "profiles", name)
     if not os.path.exists(p):
         return None
     for line in open(p):
-        if line.startswith("dram_bytes_per_full_launch:"):
+        if line.startswith(key + ":"):
             try:
                 return float(line.split(":", 1)[1].split()[0])
             except ValueError:
                 return None
     return None
+
+
+def traffic_from_profile():
+    """DRAM bytes per launch of the affinity kernel from the committed ncu summary."""
+    return profile_field("dram_bytes_per_full_launch")
 
 
 class Clocks:
@@ -188,6 +194,45 @@ def cpu_baseline(w, A_gpu, budget_s: float):
             "sample": f"affinity on {T_slice} of {w.T} tokens of one layer (fp64); "
                       f"search on the GPU's A took {1e3 * t_search:.1f} ms",
             "search_ms": 1e3 * t_search}
+
+
+# token slices on which the oracle is timed for each workload (the full tiny config; 256 tokens of one
+# layer of the Qwen-shaped and Danube-shaped models; 64 tokens of the Llama-shaped layer)
+ORACLE_SLICES = (("tiny", 256), ("qwen3_0.6b_layer", 256), ("qwen3_0.6b_model", 256),
+                 ("danube3_500m_model", 256), ("llama3.1_8b_layer", 64))
+
+
+def oracle_per_config():
+    """The fp64 oracle's affinity time per token on a token slice of every workload (layer 0)."""
+    import oracle
+    out = {}
+    for name, T in ORACLE_SLICES:
+        wc = synth.WORKLOADS[name]
+        L = synth.make_workload_layer(wc, T=T)
+        X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
+        t0 = time.perf_counter()
+        oracle.affinity_fo(X, C, Wg, Wu)
+        dt = time.perf_counter() - t0
+        out[name] = {"tokens": T, "s_per_token": dt / T, "tokens_per_s": T / dt,
+                     "gflops": flop_per_token(wc) * T / dt / 1e9}
+    return out
+
+
+def oracle_model_search(A_model, gpu_results, iters):
+    """The oracle's up-edge coordinate ascent over every layer of the model on the GPU's affinities,
+    timed on the host, per device count; also whether its layouts equal the GPU's bit for bit."""
+    import oracle
+    out = {}
+    for D, ref in gpu_results.items():
+        t0 = time.perf_counter()
+        res = [oracle.search_layout(A_model[i], D, iters) for i in range(A_model.shape[0])]
+        dt = time.perf_counter() - t0
+        same = all(r["score_q"] == int(ref["score_q"][i]) and np.array_equal(r["h"], ref["h"][i]) and
+                   np.array_equal(r["nu"], ref["nu"][i]) for i, r in enumerate(res))
+        out[f"D{D}_host_ms"] = 1e3 * dt
+        out[f"D{D}_host_matches_gpu"] = bool(same)
+    out["host_cores"] = oracle.num_threads()
+    return out
 
 
 def layout_suite(args, w, S_up, S_down, S_add, stream):
@@ -410,6 +455,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--cpu-tokens", type=int, default=64, help="token slice per step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sustained-s", type=float, default=2.0,
+                    help="seconds of back-to-back steps for the sustained figure (0: skip)")
     ap.add_argument("--model", default=None, help="time a whole-model pipeline instead, e.g. qwen3_0.6b_model")
     ap.add_argument("--add-score", action="store_true", help="with --model: also the ADD affinity and its layout")
     ap.add_argument("--producer", action="store_true",
@@ -511,6 +558,30 @@ def main():
     value = world * w.T * args.steps / (elapsed_ms / 1e3)
     clocks = clk.summary()
 
+    # sustained: the same pipelined step back to back for about --sustained-s seconds (power-capped
+    # steady state), timed on the device; the affinity launches of its second half give the
+    # sustained kernel rate, compared with cuBLAS's sustained figure
+    sus = None
+    if args.sustained_s > 0:
+        n_sus = max(10, int(args.sustained_s * 1e3 / ms_step))
+        aff_ev.clear()
+        barrier()
+        torch.cuda.synchronize()
+        with Clocks(local) as clk_s:
+            u0, u1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            u0.record(stream)
+            for k in range(n_sus):
+                step(record=k >= n_sus // 2)
+            stream.wait_stream(side)
+            u1.record(stream)
+            torch.cuda.synchronize()
+        barrier()
+        sus_ms = shard.max_over_ranks(u0.elapsed_time(u1), device=dev)
+        sus_aff = float(np.mean([a.elapsed_time(b) for a, b in aff_ev]))
+        sus = {"seconds": sus_ms / 1e3, "steps": n_sus, "value": world * w.T * n_sus / (sus_ms / 1e3),
+               "unit": UNIT, "affinity_ms_second_half": sus_aff, "clocks": clk_s.summary()}
+        aff_ev.clear()
+
     # search alone (same A, same launch) for the "search ms" part of the metric
     s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s0.record(stream)
@@ -529,6 +600,7 @@ def main():
         dtp.affinity_accumulate(Li["X"], Li["C"], Li["W_gate"], Li["W_up"], A=A_model[i])
         del Li
     model_search = {"layers": model.layers, "tokens_per_layer_for_A": 1024, "iters": model.iters}
+    model_gpu = {}
     for Dm in model.D:
         wsm = torch.empty(dtp.search_workspace_size(model.layers, model.G, model.N, Dm), dtype=torch.uint8, device=dev)
         rm = dtp.search_layout_batched(A_model, Dm, model.iters, workspace=wsm)
@@ -554,6 +626,8 @@ def main():
         model_search[f"D{Dm}_global_mean_score"] = float(rg["score"].mean())
         model_search[f"D{Dm}_ascent_over_global_min"] = float((rm["score_q"].double() / rg["score_q"].double()).min())
         model_search[f"D{Dm}_layers_at_global"] = int((rm["score_q"] == rg["score_q"]).sum())
+        model_gpu[Dm] = {k: rm[k].cpu().numpy() for k in ("h", "nu", "score_q")}
+    A_model_host = A_model.cpu().numpy()
     del A_model
 
     # ---- end to end through the public API, host buffers in pinned memory.  Every step copies its
@@ -694,7 +768,20 @@ def main():
                 "frac": achieved / peaks["bf16"], "traffic": traffic_from_profile(),
                 "kernel": "affinity_fo_tc_kernel (+ its partial-sum reduce)",
                 "peak_source": f"{peaks['source']} bf16 burst (cuBLAS 8192^3)",
-                "frac_of_sustained": achieved / peaks["bf16_sustained"] if peaks["bf16_sustained"] else None}
+                "frac_of_sustained": achieved / peaks["bf16_sustained"] if peaks["bf16_sustained"] else None,
+                # share of the kernel's active cycles with the tensor pipe busy (committed ncu summary)
+                "tensor_pipe_active_pct": profile_field("tensor_pipe_active_pct_of_active")}
+    if peaks.get("sm_mhz") and clocks.get("sm_mhz"):
+        # the peak scaled to the bench's own median SM clock: peak x (bench MHz / the peak run's MHz)
+        scale = clocks["sm_mhz"] / peaks["sm_mhz"]
+        roofline["frac_clock_normalised"] = achieved / (peaks["bf16"] * scale)
+        roofline["clock_normalisation"] = (f"peak x {clocks['sm_mhz']:.0f} MHz (bench median) / "
+                                           f"{peaks['sm_mhz']:.0f} MHz (median SM clock of the peak run)")
+    if sus is not None:
+        sus_tf = fl / (sus["affinity_ms_second_half"] / 1e3) / 1e12
+        sus["affinity_tflops"] = sus_tf
+        sus["frac_of_sustained_peak"] = sus_tf / peaks["bf16_sustained"] if peaks["bf16_sustained"] else None
+        roofline["sustained"] = sus
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
@@ -716,7 +803,12 @@ def main():
         "clocks": clocks,
     }
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, A, args.cpu_budget)
+        cb = cpu_baseline(w, A, args.cpu_budget)
+        cb["per_config"] = oracle_per_config()
+        cb["sample"] += ("; per_config: the oracle's affinity on a token slice of every workload; the 28-layer "
+                         "model search on the host on the GPU's affinities (model_search.D*_host_ms)")
+        model_search.update(oracle_model_search(A_model_host, model_gpu, model.iters))
+        line["cpu_baseline"] = cb
     print(json.dumps(line), flush=True)
 
 
