@@ -10,7 +10,11 @@
 //   gather_rows_kernel   dst block b of rows = src block perm[b]  (q/k/v rows,
 //                        gate/up rows)
 //   gather_cols_kernel   dst column block b = src column block perm[b] in
-//                        every row  (o columns, down columns)
+//                        every row  (o columns; element-wise columns whose
+//                        rows are not a multiple of 16 bytes)
+//   gather_cols_staged_kernel  the same for element-wise columns (down
+//                        columns, one per neuron) with 16-byte rows: row tiles
+//                        and the permutation staged in shared memory
 // The gathers are pure data movement, bound by HBM: every byte is read once
 // and written once with 16-byte accesses where the block width allows it.  A
 // permutation entry outside [0, blocks) is not followed: the element is left
@@ -197,6 +201,164 @@ __global__ void gather_cols_kernel(const uint8_t* __restrict__ src, uint8_t* __r
     }
 }
 
+// Element-wise column gather staged through shared memory (rows of a multiple
+// of 16 bytes whose column blocks are not whole 16-byte words, e.g. one
+// down_proj column per neuron).  Gathering such elements straight from global
+// memory costs one 32-byte L1 sector per element; here each CTA
+//   - copies its layer's permutation into shared memory once,
+//   - streams tiles of R consecutive rows (contiguous in memory) into a ring of
+//     kStagedStages shared buffers with 1-D bulk copies (cp.async.bulk,
+//     completion counted on an mbarrier), one thread issuing them,
+//   - lets each thread own a fixed set of 16-byte output words: it turns the
+//     permutation entries behind a word into shared-memory offsets once per
+//     tile, then walks the tile's rows gathering from shared memory (4-byte
+//     banks) and storing 16-byte words, coalesced across the warp.
+// CTAs take contiguous ranges of the layers x row-tiles list, so a CTA loads
+// a new permutation only when its range crosses into the next layer.  Small
+// CTAs with two stages keep several CTAs per SM and enough bulk copies in
+// flight; tiles of about 16 KB amortise the per-tile barrier.
+constexpr int kStagedThreads = 128;
+constexpr int kStagedStages = 2;
+constexpr int64_t kStagedTileTarget = 16 * 1024;   // bytes per staged row tile (at least one row)
+
+struct StagedGeom {
+    int64_t rows, row_bytes, block_elems, nblocks, perm_stride;
+    int layers, tile_rows, tiles_per_layer;
+    int64_t total_tiles;
+};
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+template <typename E>
+__global__ void __launch_bounds__(kStagedThreads)
+gather_cols_staged_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst, StagedGeom g,
+                          const int32_t* __restrict__ perm, int* status) {
+    constexpr int kPer = static_cast<int>(16 / sizeof(E));
+    constexpr uint32_t kNone = 0xFFFFFFFFu;            // offset of an entry that is not followed
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(8) uint64_t bars[kStagedStages];
+    __shared__ int abort_flag;
+    const uint32_t row_bytes = static_cast<uint32_t>(g.row_bytes);
+    const uint32_t stage_bytes = static_cast<uint32_t>(g.tile_rows) * row_bytes;
+    int32_t* perm_s = reinterpret_cast<int32_t*>(smem + kStagedStages * stage_bytes);
+    const int tid = threadIdx.x;
+    // this CTA's contiguous range of (layer, row tile) items
+    const int64_t t_begin = g.total_tiles * blockIdx.x / gridDim.x;
+    const int64_t t_end = g.total_tiles * (blockIdx.x + 1) / gridDim.x;
+    if (t_begin >= t_end) return;
+    if (tid == 0) {
+        abort_flag = 0;
+        for (int i = 0; i < kStagedStages; ++i) mbar_init(smem_u32(&bars[i]), 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+
+    auto tile_rows_of = [&](int64_t t) -> int {
+        const int64_t r0 = (t % g.tiles_per_layer) * g.tile_rows;
+        return static_cast<int>(min(static_cast<int64_t>(g.tile_rows), g.rows - r0));
+    };
+    auto issue = [&](int64_t t) {      // tile t into stage (t - t_begin) % S
+        const int64_t layer = t / g.tiles_per_layer;
+        const int64_t r0 = (t % g.tiles_per_layer) * g.tile_rows;
+        const uint32_t bytes = static_cast<uint32_t>(tile_rows_of(t)) * row_bytes;
+        const int st = static_cast<int>((t - t_begin) % kStagedStages);
+        const uint32_t bar = smem_u32(&bars[st]);
+        mbar_arrive_expect_tx(bar, bytes);
+        bulk_g2s(smem_u32(smem + st * stage_bytes), src + (layer * g.rows + r0) * g.row_bytes, bytes, bar);
+    };
+    if (tid == 0)
+        for (int64_t t = t_begin; t < t_end && t < t_begin + kStagedStages; ++t) issue(t);
+
+    int64_t cur_layer = -1;
+    int bad = 0;
+    const int words = static_cast<int>(g.row_bytes / 16);
+    const uint32_t be = static_cast<uint32_t>(g.block_elems);
+    const uint32_t nblocks = static_cast<uint32_t>(g.nblocks);
+    int64_t t = t_begin;
+    for (; t < t_end; ++t) {
+        const int64_t layer = t / g.tiles_per_layer;
+        if (layer != cur_layer) {      // (re)load the layer's permutation; nobody reads perm_s here
+            const int32_t* pl = perm + layer * g.perm_stride;
+            for (int64_t b = tid; b < g.nblocks; b += kStagedThreads) perm_s[b] = pl[b];
+            cur_layer = layer;
+            __syncthreads();
+        }
+        const int st = static_cast<int>((t - t_begin) % kStagedStages);
+        const uint32_t parity = static_cast<uint32_t>(((t - t_begin) / kStagedStages) & 1);
+        // the block leaves together: a wait that gave up makes every thread's wait give up
+        // (shared abort flag), and the vote keeps the barrier counts of all threads equal
+        const bool landed = mbar_wait(smem_u32(&bars[st]), parity, &abort_flag);
+        if (!__syncthreads_and(landed)) break;
+        const uint8_t* tile = smem + st * stage_bytes;
+        const int nr = tile_rows_of(t);
+        const int64_t r0 = (t % g.tiles_per_layer) * g.tile_rows;
+        uint8_t* out = dst + (layer * g.rows + r0) * g.row_bytes;
+        for (int ow = tid; ow < words; ow += kStagedThreads) {
+            // byte offsets in a staged row of the kPer source elements behind output word ow
+            uint32_t off[kPer];
+            if (kPer % 4 == 0 && be == 1) {
+                const int4* pv = reinterpret_cast<const int4*>(perm_s + ow * kPer);
+#pragma unroll
+                for (int q = 0; q < kPer / 4; ++q) {
+                    const int4 p4 = pv[q];
+                    const int32_t pe[4] = {p4.x, p4.y, p4.z, p4.w};
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const bool ok = static_cast<uint32_t>(pe[k]) < nblocks;
+                        bad |= !ok;
+                        off[4 * q + k] = ok ? static_cast<uint32_t>(pe[k]) * sizeof(E) : kNone;
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < kPer; ++i) {
+                    const uint32_t c = static_cast<uint32_t>(ow) * kPer + i;
+                    const uint32_t b = c / be;
+                    const int32_t pb = perm_s[b];
+                    const bool ok = static_cast<uint32_t>(pb) < nblocks;
+                    bad |= !ok;
+                    off[i] = ok ? (static_cast<uint32_t>(pb) * be + (c - b * be)) * sizeof(E) : kNone;
+                }
+            }
+            const uint8_t* rowp = tile;
+            uint8_t* op = out + static_cast<int64_t>(ow) * 16;
+#pragma unroll 2
+            for (int r = 0; r < nr; ++r) {
+                union { uint4 v; E e[kPer]; } w;
+#pragma unroll
+                for (int i = 0; i < kPer; ++i)
+                    w.e[i] = off[i] != kNone ? *reinterpret_cast<const E*>(rowp + off[i]) : E(0);
+                *reinterpret_cast<uint4*>(op) = w.v;
+                rowp += row_bytes;
+                op += g.row_bytes;
+            }
+        }
+        // every thread is done with this stage (and with perm_s before a reload): refill it
+        __syncthreads();
+        if (tid == 0 && t + kStagedStages < t_end) issue(t + kStagedStages);
+    }
+    if (bad) atomicMin(status, static_cast<int>(DTP_ERR_ARG));
+    if (t < t_end) {
+        // a wait gave up: report it, then let the copies still in flight land before exiting
+        __syncthreads();
+        if (tid == 0) {
+            atomicMin(status, static_cast<int>(DTP_ERR_NOT_CONVERGED));
+            int ok = 1;
+            for (int64_t u = t; u < t_end && u < t + kStagedStages && ok; ++u) {
+                volatile int own = 0;
+                const int su = static_cast<int>((u - t_begin) % kStagedStages);
+                ok = mbar_wait(smem_u32(&bars[su]), static_cast<uint32_t>(((u - t_begin) / kStagedStages) & 1), &own);
+            }
+        }
+        __syncthreads();
+    }
+}
+
 static int grid_for(int64_t work) {
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
@@ -251,6 +413,66 @@ static void cols_by_elem(const uint8_t* s, uint8_t* d, int layers, int64_t rows,
                                                                 perm_stride, status);
 }
 
+// Element-wise path straight from global memory, for any element width.
+static void cols_by_elem_any(const uint8_t* s, uint8_t* d, int layers, int64_t rows, int64_t row_bytes,
+                             int64_t block_bytes, int elem_bytes, const int32_t* perm, int64_t perm_stride,
+                             int* status, int grid, bool pack, cudaStream_t stream) {
+    if (elem_bytes == 2)
+        cols_by_elem<uint16_t>(s, d, layers, rows, row_bytes, block_bytes, perm, perm_stride, status, grid, pack, stream);
+    else if (elem_bytes == 4)
+        cols_by_elem<uint32_t>(s, d, layers, rows, row_bytes, block_bytes, perm, perm_stride, status, grid, pack, stream);
+    else if (elem_bytes == 8)
+        cols_by_elem<uint64_t>(s, d, layers, rows, row_bytes, block_bytes, perm, perm_stride, status, grid, pack, stream);
+    else
+        cols_by_elem<uint8_t>(s, d, layers, rows, row_bytes, block_bytes, perm, perm_stride, status, grid, pack, stream);
+}
+
+template <typename E>
+static int launch_staged_as(const uint8_t* s, uint8_t* d, const StagedGeom& g, size_t smem, const int32_t* perm,
+                            int* status, cudaStream_t stream) {
+    auto* fn = gather_cols_staged_kernel<E>;
+    DTP_CUDA_TRY(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
+    int dev = 0, sms = 0, per_sm = 0;
+    DTP_CUDA_TRY(cudaGetDevice(&dev));
+    DTP_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    DTP_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kStagedThreads, smem));
+    if (per_sm < 1) return DTP_ERR_UNSUPPORTED;
+    const int64_t cap = static_cast<int64_t>(sms) * per_sm;
+    const int grid = static_cast<int>(g.total_tiles < cap ? g.total_tiles : cap);
+    fn<<<grid, kStagedThreads, smem, stream>>>(s, d, g, perm, status);
+    DTP_CUDA_TRY(cudaGetLastError());
+    return DTP_OK;
+}
+
+// Returns DTP_ERR_UNSUPPORTED (nothing launched) when a permutation and the
+// stages do not fit in shared memory; the caller then gathers from global memory.
+static int launch_cols_staged(const uint8_t* s, uint8_t* d, int layers, int64_t rows, int64_t row_bytes,
+                              int64_t block_elems, int elem_bytes, const int32_t* perm, int64_t perm_stride,
+                              int* status, cudaStream_t stream) {
+    StagedGeom g;
+    g.rows = rows;
+    g.row_bytes = row_bytes;
+    g.block_elems = block_elems;
+    g.nblocks = row_bytes / elem_bytes / block_elems;
+    g.perm_stride = perm_stride;
+    g.layers = layers;
+    int64_t tr = kStagedTileTarget / row_bytes;
+    if (tr < 1) tr = 1;
+    if (tr > rows) tr = rows;
+    g.tile_rows = static_cast<int>(tr);
+    g.tiles_per_layer = static_cast<int>((rows + tr - 1) / tr);
+    g.total_tiles = static_cast<int64_t>(layers) * g.tiles_per_layer;
+    const size_t smem = static_cast<size_t>(kStagedStages) * static_cast<size_t>(tr * row_bytes) +
+                        align_up(static_cast<size_t>(g.nblocks) * 4, 16);
+    if (smem > 200 * 1024 || tr * row_bytes > (int64_t(1) << 30) || g.total_tiles < 1) return DTP_ERR_UNSUPPORTED;
+    switch (elem_bytes) {
+        case 1: return launch_staged_as<uint8_t>(s, d, g, smem, perm, status, stream);
+        case 2: return launch_staged_as<uint16_t>(s, d, g, smem, perm, status, stream);
+        case 4: return launch_staged_as<uint32_t>(s, d, g, smem, perm, status, stream);
+        default: return launch_staged_as<uint64_t>(s, d, g, smem, perm, status, stream);
+    }
+}
+
 int launch_cols(const void* src, void* dst, int layers, int64_t rows, int64_t row_bytes, int64_t block_bytes,
                 int elem_bytes, const int32_t* perm, int64_t perm_stride, void* workspace, cudaStream_t stream) {
     int* status = reinterpret_cast<int*>(workspace);
@@ -263,6 +485,13 @@ int launch_cols(const void* src, void* dst, int layers, int64_t rows, int64_t ro
     if (rows16 && block_bytes % 16 == 0) {
         gather_cols_kernel<uint4, kDirect><<<grid, 256, 0, stream>>>(s, d, layers, rows, row_bytes, block_bytes, perm,
                                                                      perm_stride, status);
+    } else if (rows16 && (elem_bytes == 1 || elem_bytes == 2 || elem_bytes == 4 || elem_bytes == 8) &&
+               (mis & (elem_bytes - 1)) == 0 && block_bytes % elem_bytes == 0) {
+        const int st = launch_cols_staged(s, d, layers, rows, row_bytes, block_bytes / elem_bytes, elem_bytes, perm,
+                                          perm_stride, status, stream);
+        if (st != DTP_ERR_UNSUPPORTED) return st;
+        cols_by_elem_any(s, d, layers, rows, row_bytes, block_bytes, elem_bytes, perm, perm_stride, status, grid,
+                         rows16, stream);
     } else if (elem_bytes == 2 && (mis & 1) == 0) {
         cols_by_elem<uint16_t>(s, d, layers, rows, row_bytes, block_bytes, perm, perm_stride, status, grid, rows16,
                                stream);

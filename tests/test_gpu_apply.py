@@ -153,7 +153,8 @@ def test_permute_rejects_out_of_range_entries():
 
 @pytest.mark.parametrize("dtype,rows,cols,block", [
     (torch.float32, 64, 96, 1), (torch.float32, 40, 30, 3), (torch.bfloat16, 33, 3072, 1),
-    (torch.bfloat16, 16, 24, 8), (torch.uint8, 10, 48, 3), (torch.uint8, 7, 21, 7), (torch.float64, 9, 12, 2)])
+    (torch.bfloat16, 16, 24, 8), (torch.uint8, 10, 48, 3), (torch.uint8, 7, 21, 7), (torch.float64, 9, 12, 2),
+    (torch.float64, 8, 14, 1), (torch.uint8, 12, 64, 1), (torch.bfloat16, 5, 14336, 1), (torch.float32, 3, 4100, 2)])
 def test_gathers_match_indexing(dtype, rows, cols, block):
     """Every width path of the gathers (16-byte words, packed elements, plain elements) against
     plain indexing, on two stacked layers with different permutations."""
@@ -180,3 +181,16 @@ def test_staged_column_gather_rejects_out_of_range_entries():
     with pytest.raises(dtp.DTPError) as e:
         dtp.permute_cols(src, perm, 1)
     assert e.value.status == dtp.DTP_ERR_ARG
+
+
+@pytest.mark.parametrize("layers,rows,cols", [(28, 1024, 3072), (1, 4096, 14336), (16, 1536, 4096)])
+def test_down_column_gather_at_model_size(layers, rows, cols):
+    """The down_proj column gather (one column per neuron, rows staged in shared memory) at the
+    Qwen3-0.6B (28 layers), Llama-3.1-8B and Danube3-500M shapes: bit-exact against indexing."""
+    g = torch.Generator(device=DEV).manual_seed(cols)
+    src = torch.randn((layers, rows, cols), device=DEV, generator=g).to(torch.bfloat16)
+    perm = torch.stack([torch.randperm(cols, device=DEV, generator=g) for _ in range(layers)]).to(torch.int32)
+    got = dtp.permute_cols(src, perm, 1)
+    ref = torch.gather(src, 2, perm.long().unsqueeze(1).expand(layers, rows, cols))
+    assert torch.equal(got, ref)
+
