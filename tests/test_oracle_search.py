@@ -148,6 +148,54 @@ def test_neuron_step_matches_hungarian(N, D):
             assert sorted(r2c.tolist()) == list(range(N))
 
 
+def _lex_smallest_by_fixing(q, h, D):
+    """The lexicographically smallest optimal balanced assignment, straight from its definition:
+    for k = 0, 1, ... give neuron k the smallest device with which the optimum total is still
+    reachable, each test a textbook Hungarian solve of the slot-expanded matrix in which the rows of
+    the neurons fixed so far keep only their device's slots.  The optimum is unique exactly when
+    every step finds a single such device (a second optimum differs from the lexicographically
+    smallest one first at some neuron k, and agrees with it before k)."""
+    G, N = q.shape
+    M = np.zeros((N, D), dtype=np.int64)
+    for g in range(G):
+        M[:, h[g]] += q[g]
+    cap = N // D
+    W = np.repeat(M, cap, axis=1)
+    best, _ = oracle.hungarian_max(W)
+    penalty = -(1 << 50)                 # far below any total the scores can reach (< 2^47 here)
+    nu = np.zeros(N, dtype=np.int32)
+    unique = True
+    for k in range(N):
+        keep = []
+        for l in range(D):
+            trial = W.copy()
+            trial[k, :] = penalty
+            trial[k, l * cap:(l + 1) * cap] = W[k, l * cap:(l + 1) * cap]
+            if oracle.hungarian_max(trial)[0] == best:
+                keep.append((l, trial))
+        assert keep, "no device keeps the optimum"
+        unique &= len(keep) == 1
+        nu[k], W = keep[0]
+    return nu, best, unique
+
+
+@pytest.mark.parametrize("G,N,D", [(8, 48, 4), (8, 96, 3), (6, 60, 3), (8, 64, 8), (4, 40, 2), (8, 72, 4)])
+def test_neuron_step_tie_break_by_fixing(G, N, D):
+    """The oracle's lexicographic tie-break (successive shortest paths, then LP duality and Hall's
+    condition) and its uniqueness flag against the plain definition of the lexicographically smallest
+    optimum, on tie-heavy integer scores far beyond brute-force sizes (Sec. 3 "Optimiser"; ties to
+    the lowest index), and on continuous scores with a unique optimum."""
+    h = np.array([(g * D) // G for g in range(G)] if G % D == 0 else [g % D for g in range(G)], dtype=np.int32)
+    for seed, kind in ((0, "integer"), (1, "integer"), (2, "lognormal")):
+        _, q = _rand_q(G, N, 500 + 10 * seed + N + D, kind)
+        ref, best, ref_unique = _lex_smallest_by_fixing(q, h, D)
+        for general in (False, True):
+            nu, uniq = oracle.neuron_step(q, h, D, general=general)
+            assert oracle.assignment_gain(q, h, nu, D) == best
+            np.testing.assert_array_equal(nu, ref)
+            assert uniq == ref_unique
+
+
 def _qwen_layer_q(layer, T=64):
     """Exact scores of a Qwen3-0.6B-shaped layer (G = 8, N = 3072) from the oracle's affinity on a
     token slice of that layer's synthetic activations."""
