@@ -348,6 +348,8 @@ def run_model(args):
     t_prod = 0.0
     if args.producer and q not in (1, w.q_per_group):
         raise SystemExit("--producer takes --qheads 1 (KV-group rows) or the model's query heads per group")
+    clk = Clocks(local)
+    clk.__enter__()
     for li, i in enumerate(mine):
         L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
             synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
@@ -395,6 +397,7 @@ def run_model(args):
         if args.add_score:
             t_add += e2.elapsed_time(e3)
         del L, Dn
+    clk.__exit__(None, None, None)
     if dtp.workspace_status(ws) != dtp.DTP_OK:
         raise RuntimeError("affinity kernel reported a device-side error")
     torch.cuda.synchronize()
@@ -442,7 +445,9 @@ def run_model(args):
                                 "uniform": 1.0 / G},
             "pipeline_s": (total_ms + suite["ms"] + apply["ms"]) / 1e3,
             "producer_ms": t_prod if args.producer else None,
-            "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s"}
+            "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s",
+            "clocks": clk.summary(),
+            "clocks_note": "sampled over the per-layer scoring loop (input generation included)"}
     print(json.dumps(line), flush=True)
 
 
