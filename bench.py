@@ -776,17 +776,19 @@ def main():
                 "frac_of_sustained": achieved / peaks["bf16_sustained"] if peaks["bf16_sustained"] else None,
                 # share of the kernel's active cycles with the tensor pipe busy (committed ncu summary)
                 "tensor_pipe_active_pct": profile_field("tensor_pipe_active_pct_of_active")}
-    if peaks.get("sm_mhz") and clocks.get("sm_mhz"):
-        # the peak scaled to the bench's own median SM clock: peak x (bench MHz / the peak run's MHz)
-        scale = clocks["sm_mhz"] / peaks["sm_mhz"]
-        roofline["frac_clock_normalised"] = achieved / (peaks["bf16"] * scale)
-        roofline["clock_normalisation"] = (f"peak x {clocks['sm_mhz']:.0f} MHz (bench median) / "
-                                           f"{peaks['sm_mhz']:.0f} MHz (median SM clock of the peak run)")
     if sus is not None:
         sus_tf = fl / (sus["affinity_ms_second_half"] / 1e3) / 1e12
         sus["affinity_tflops"] = sus_tf
         sus["frac_of_sustained_peak"] = sus_tf / peaks["bf16_sustained"] if peaks["bf16_sustained"] else None
         roofline["sustained"] = sus
+        sus_mhz = sus["clocks"].get("sm_mhz")
+        if peaks.get("sm_mhz") and sus_mhz and peaks["bf16_sustained"]:
+            # work per SM clock cycle, the sustained affinity kernel against cuBLAS's sustained loop;
+            # the peak file's median SM clock was sampled over that loop, so the two are like for like
+            roofline["frac_clock_normalised"] = (sus_tf / sus_mhz) / (peaks["bf16_sustained"] / peaks["sm_mhz"])
+            roofline["clock_normalisation"] = (
+                f"(sustained {sus_tf:.0f} TFLOP/s / {sus_mhz:.0f} MHz median) / (cuBLAS sustained "
+                f"{peaks['bf16_sustained']:.0f} TFLOP/s / {peaks['sm_mhz']:.0f} MHz median under load)")
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
