@@ -11,13 +11,19 @@
 //
 // A GEMM with a short K (Kj = 96..512) whose output (T x d per row, bf16) is
 // far larger than its inputs: the kernel is bound by the HBM write of C.
-// Persistent grid, one CTA per SM.  Warp 0 loads 128 x 64 tiles of attn and
-// 256 x 64 tiles of W_o by TMA, warp 1 issues 128 x 256 x 16 tcgen05.mma into
-// a double-buffered TMEM accumulator, eight epilogue warps (lane quadrant x
-// column half) scale by gamma / r in fp32, round to bf16 and write 32 x 64
-// boxes through 128B-swizzled staging buffers with TMA bulk stores.  Units are
-// ordered with the 256-column tile fastest, so each 128-token tile of attn is
-// read from HBM once and reused from L2 for every column tile.
+// Persistent grid, one CTA per SM, 20 warps.  Warp 0 loads 128 x 64 tiles of
+// attn and 256 x 64 tiles of W_o by TMA, warp 1 issues 128 x 256 x 16
+// tcgen05.mma into a double-buffered TMEM accumulator, and sixteen epilogue
+// warps in two sets of eight drain it: set 0 takes the CTA's even units
+// (TMEM buffer 0), set 1 the odd ones (buffer 1), so one set's TMEM loads and
+// scaling overlap the other's stores.  An epilogue warp owns 32 tokens (its
+// TMEM lane quadrant) x 128 columns and writes them as four 32 x 32 bf16
+// boxes: scale by gamma / r in fp32 (packed f32x2 multiplies), round to bf16,
+// store into a 64-byte-swizzled staging buffer and issue a TMA bulk store
+// (two staging buffers per warp).  Boxes of 32 columns keep a thread's
+// registers under the 102 that 640 threads allow.  Units are ordered with the
+// 256-column tile fastest, so each 128-token tile of attn is read from HBM
+// once and reused from L2 for every column tile.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -34,13 +40,13 @@ constexpr int BC = 256;       // output columns per tile (MMA N)
 constexpr int BK = 64;
 constexpr int UK = 16;
 constexpr int STAGES = 3;
-constexpr int kThreads = 384;
-constexpr int kEpiWarps = 8;
+constexpr int kThreads = 640;
+constexpr int kEpiWarps = 16;   // two sets of 8, one per TMEM buffer
 constexpr int kEpiWarp0 = 4;
 constexpr uint32_t kTileA = BT * BK * 2;          // 16 KB
 constexpr uint32_t kTileB = BC * BK * 2;          // 32 KB
 constexpr uint32_t kStageBytes = kTileA + kTileB;
-constexpr uint32_t kStageOut = 32 * 128;          // one 32-row x 64-column bf16 box, 4 KB
+constexpr uint32_t kStageOut = 32 * 64;           // one 32-row x 32-column bf16 box, 2 KB (64-byte swizzle)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kBufCols = 256;
 constexpr size_t kSmemBytes = 1024 + STAGES * kStageBytes + kEpiWarps * 2 * kStageOut + 256;
@@ -70,6 +76,16 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Two fp32 products in one packed instruction (mul.rn.f32x2): each lane rounds as a scalar
+// mul.rn.f32 does.
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
@@ -110,7 +126,7 @@ head_writes_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_con
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
-            mbar_init(smem_u32(&acc_empty[b]), kEpiWarps);
+            mbar_init(smem_u32(&acc_empty[b]), kEpiWarps / 2);
         }
         mbar_init(smem_u32(drain_bar), 1);
         *abort_flag = 0;
@@ -197,54 +213,64 @@ head_writes_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_con
         }
     } else if (warp >= kEpiWarp0) {
         // -------------------------------------------------------------------- epilogue
+        // set 0 takes the CTA's even units (TMEM buffer 0), set 1 the odd ones (buffer 1), so one
+        // set's TMEM loads and scaling overlap the other's stores
+        const int set = (warp - kEpiWarp0) >> 3;
         const int quad = warp & 3;                      // TMEM lanes 32*quad .. (tokens)
-        const int half = (warp - kEpiWarp0) >> 2;       // columns 128*half .. of the tile
+        const int half = ((warp - kEpiWarp0) >> 2) & 1; // columns 128*half .. of the tile
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
         uint8_t* stg = staging + (warp - kEpiWarp0) * 2 * kStageOut;
-        uint32_t sbuf = 0, unit_count = 0;
+        uint32_t sbuf = 0;
         bool ok = true;
-        for (int64_t u = blockIdx.x; ok && u < p.units; u += gridDim.x, ++unit_count) {
+        const uint32_t buf = static_cast<uint32_t>(set);
+        for (int64_t k = set;; k += 2) {
+            const int64_t u = blockIdx.x + k * gridDim.x;
+            if (!ok || u >= p.units) break;
             int j, tt, dc;
             decode(p, u, j, tt, dc);
-            const uint32_t buf = unit_count & 1u;
-            const uint32_t use = (unit_count >> 1) & 1u;
+            const uint32_t use = static_cast<uint32_t>((k >> 1) & 1);
             if (!mbar_wait(smem_u32(&acc_full[buf]), use, abort_flag)) { ok = false; break; }
             tc_fence_after();
             const int64_t t = static_cast<int64_t>(tt) * BT + quad * 32 + lane;
             const float rinv = t < p.T ? 1.0f / p.rms[t] : 0.0f;
+            const float2 rr = make_float2(rinv, rinv);
             const int y0 = tt * BT + quad * 32;
             const uint32_t acc = lane_base + buf * kBufCols;
 #pragma unroll 1
-            for (int c = 0; c < 2; ++c) {
-                const int col0 = 128 * half + 64 * c;
+            for (int c = 0; c < 4; ++c) {
+                const int col0 = 128 * half + 32 * c;
                 const int g0 = dc * BC + col0;
                 if (g0 >= p.d || y0 >= p.T) continue;   // box entirely outside C (warp-uniform)
-                float v[64];
+                float4 gm[8];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) tmem_ld16(acc + static_cast<uint32_t>(col0 + 16 * q), &v[16 * q]);
+                for (int q = 0; q < 8; ++q)
+                    gm[q] = g0 + 4 * q < p.d ? __ldg(reinterpret_cast<const float4*>(p.gamma + g0) + q)
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+                float v[32];
+                tmem_ld16(acc + static_cast<uint32_t>(col0), &v[0]);
+                tmem_ld16(acc + static_cast<uint32_t>(col0 + 16), &v[16]);
                 tmem_wait_ld();
 #pragma unroll
-                for (int e = 0; e < 64; e += 4) {
-                    float4 gm = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (g0 + e < p.d) gm = __ldg(reinterpret_cast<const float4*>(p.gamma + g0 + e));
-                    v[e] *= gm.x * rinv;
-                    v[e + 1] *= gm.y * rinv;
-                    v[e + 2] *= gm.z * rinv;
-                    v[e + 3] *= gm.w * rinv;
+                for (int q = 0; q < 8; ++q) {
+                    const float2 s01 = mul2(make_float2(gm[q].x, gm[q].y), rr);
+                    const float2 s23 = mul2(make_float2(gm[q].z, gm[q].w), rr);
+                    const float2 a = mul2(make_float2(v[4 * q], v[4 * q + 1]), s01);
+                    const float2 b = mul2(make_float2(v[4 * q + 2], v[4 * q + 3]), s23);
+                    v[4 * q] = a.x; v[4 * q + 1] = a.y; v[4 * q + 2] = b.x; v[4 * q + 3] = b.y;
                 }
                 // the staging buffer is free once the store issued from it two boxes ago has read it
                 if (lane == 0) bulk_wait_read1();
                 __syncwarp();
                 uint8_t* sb = stg + sbuf * kStageOut;
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
+                for (int cc = 0; cc < 4; ++cc) {
                     uint4 w;
                     w.x = pack_bf16(v[8 * cc], v[8 * cc + 1]);
                     w.y = pack_bf16(v[8 * cc + 2], v[8 * cc + 3]);
                     w.z = pack_bf16(v[8 * cc + 4], v[8 * cc + 5]);
                     w.w = pack_bf16(v[8 * cc + 6], v[8 * cc + 7]);
-                    // 128-byte swizzle: 16-byte chunk cc of row `lane` sits at chunk cc ^ (lane & 7)
-                    *reinterpret_cast<uint4*>(sb + lane * 128 + ((cc ^ (lane & 7)) << 4)) = w;
+                    // 64-byte swizzle: 16-byte chunk cc of row `lane` sits at chunk cc ^ ((lane >> 1) & 3)
+                    *reinterpret_cast<uint4*>(sb + lane * 64 + ((cc ^ ((lane >> 1) & 3)) << 4)) = w;
                 }
                 fence_async_smem();
                 __syncwarp();
@@ -285,13 +311,13 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 static bool map_bf16(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides,
-                     cuuint32_t box_x, cuuint32_t box_y) {
+                     cuuint32_t box_x, cuuint32_t box_y, CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
     auto enc = encode_fn();
     if (!enc) return false;
     cuuint32_t box[3] = {box_x, box_y, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -307,7 +333,7 @@ int launch(const void* attn, const void* Wo, const float* gamma, const float* rm
     cuuint64_t dc[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(rows)};
     cuuint64_t sc[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(d) * 2 * static_cast<cuuint64_t>(T)};
     if (!map_bf16(&ma, attn, 2, da, sk, BK, BT) || !map_bf16(&mw, Wo, 2, dw, sk, BK, BC) ||
-        !map_bf16(&mc, C, 3, dc, sc, 64, 32))
+        !map_bf16(&mc, C, 3, dc, sc, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return DTP_ERR_CUDA;
     Params p;
     p.rows = rows;
