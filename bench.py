@@ -348,56 +348,54 @@ def run_model(args):
     t_prod = 0.0
     if args.producer and q not in (1, w.q_per_group):
         raise SystemExit("--producer takes --qheads 1 (KV-group rows) or the model's query heads per group")
-    clk = Clocks(local)
-    clk.__enter__()
-    for li, i in enumerate(mine):
-        L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
-            synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
-        if args.producer:
-            # C from the attention outputs: one row per query head, or per KV group when q == 1
-            P = synth.make_attention_inputs(T, d, G * w.q_per_group, w.head_dim, w.layer_seed(i) + 2000, device=dev)
+    with Clocks(local) as clk:
+        for li, i in enumerate(mine):
+            L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
+                synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
+            if args.producer:
+                # C from the attention outputs: one row per query head, or per KV group when q == 1
+                P = synth.make_attention_inputs(T, d, G * w.q_per_group, w.head_dim, w.layer_seed(i) + 2000, device=dev)
+                torch.cuda.synchronize()
+                p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                p0.record(stream)
+                L["C"] = dtp.head_writes(P["attn"], P["W_o"], P["gamma"], P["rms"], w.head_dim,
+                                         1 if q > 1 else w.q_per_group, out=L["C"])
+                p1.record(stream)
+                torch.cuda.synchronize()
+                t_prod += p0.elapsed_time(p1)
+                del P
+            Dn = synth.make_down_inputs(d, G, w.qkv_rows, N, T, seed=w.seed + 1000 + i, device=dev)
+            act2 = torch.zeros(N, dtype=torch.float32, device=dev)
+            A = S_up_loc[li]
+            A.zero_()
             torch.cuda.synchronize()
-            p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            p0.record(stream)
-            L["C"] = dtp.head_writes(P["attn"], P["W_o"], P["gamma"], P["rms"], w.head_dim,
-                                     1 if q > 1 else w.q_per_group, out=L["C"])
-            p1.record(stream)
-            torch.cuda.synchronize()
-            t_prod += p0.elapsed_time(p1)
-            del P
-        Dn = synth.make_down_inputs(d, G, w.qkv_rows, N, T, seed=w.seed + 1000 + i, device=dev)
-        act2 = torch.zeros(N, dtype=torch.float32, device=dev)
-        A = S_up_loc[li]
-        A.zero_()
-        torch.cuda.synchronize()
-        e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-        e0.record(stream)
-        if q == 1:
-            dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"], A=A, act2=act2,
-                                         workspace=ws)
-        else:   # one row of C per query head, summed over each KV group's q query heads
-            dtp.affinity_accumulate_grouped(L["X"], L["C"], L["W_gate"], L["W_up"], q, A=A, rms_next=Dn["rms"],
-                                            act2=act2, workspace=ws)
-        dtp.affinity_finalize(A, T, dtp.down_sqnorm(Dn["W_down"]))
-        e1.record(stream)
-        if i + 1 < Lyr:
-            bn = dtp.down_weight_sqnorm(Dn["Wqkv"], Dn["gamma"], Dn["W_down"])
-            S_down_loc[li].copy_(dtp.down_finalize(act2, bn, T))
-        e2.record(stream)
-        if args.add_score:
-            e3 = torch.cuda.Event(enable_timing=True)
+            e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            e0.record(stream)
             if q == 1:
-                dtp.affinity_add_accumulate(L["C"], L["W_gate"], L["W_up"], A_add=S_add_loc[li])
-            else:
-                dtp.affinity_add_accumulate_grouped(L["C"], L["W_gate"], L["W_up"], q, A_add=S_add_loc[li])
-            e3.record(stream)
-        torch.cuda.synchronize()
-        t_aff += e0.elapsed_time(e1)
-        t_down += e1.elapsed_time(e2)
-        if args.add_score:
-            t_add += e2.elapsed_time(e3)
-        del L, Dn
-    clk.__exit__(None, None, None)
+                dtp.affinity_accumulate_down(L["X"], L["C"], L["W_gate"], L["W_up"], Dn["rms"], A=A, act2=act2,
+                                             workspace=ws)
+            else:   # one row of C per query head, summed over each KV group's q query heads
+                dtp.affinity_accumulate_grouped(L["X"], L["C"], L["W_gate"], L["W_up"], q, A=A, rms_next=Dn["rms"],
+                                                act2=act2, workspace=ws)
+            dtp.affinity_finalize(A, T, dtp.down_sqnorm(Dn["W_down"]))
+            e1.record(stream)
+            if i + 1 < Lyr:
+                bn = dtp.down_weight_sqnorm(Dn["Wqkv"], Dn["gamma"], Dn["W_down"])
+                S_down_loc[li].copy_(dtp.down_finalize(act2, bn, T))
+            e2.record(stream)
+            if args.add_score:
+                e3 = torch.cuda.Event(enable_timing=True)
+                if q == 1:
+                    dtp.affinity_add_accumulate(L["C"], L["W_gate"], L["W_up"], A_add=S_add_loc[li])
+                else:
+                    dtp.affinity_add_accumulate_grouped(L["C"], L["W_gate"], L["W_up"], q, A_add=S_add_loc[li])
+                e3.record(stream)
+            torch.cuda.synchronize()
+            t_aff += e0.elapsed_time(e1)
+            t_down += e1.elapsed_time(e2)
+            if args.add_score:
+                t_add += e2.elapsed_time(e3)
+            del L, Dn
     if dtp.workspace_status(ws) != dtp.DTP_OK:
         raise RuntimeError("affinity kernel reported a device-side error")
     torch.cuda.synchronize()
