@@ -647,24 +647,11 @@ __global__ void affinity_reduce_rows_kernel(const float* __restrict__ partial, f
     }
 }
 
-static PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
-        void* ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    }
-    return fn;
-}
-
 // bf16 tensor map with a [box_rows x 64] box and 128-byte swizzle; out-of-range
 // elements read as zero, which contributes nothing to any sum below.
 static bool make_map(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides,
                      cuuint32_t box_rows) {
-    auto enc = get_encode_fn();
+    auto enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint32_t box[3] = {static_cast<cuuint32_t>(BK), box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};

@@ -4,8 +4,11 @@
 #pragma once
 
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <atomic>
 
 #include "dtp.h"
 
@@ -27,6 +30,24 @@ constexpr uint64_t kWaitLimitNs = 2000ull * 1000ull * 1000ull;
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// The driver's cuTensorMapEncodeTiled, looked up through the runtime once per process (a failed
+// lookup is retried on the next call).  Safe to call from several host threads at once.
+inline PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static std::atomic<PFN_cuTensorMapEncodeTiled_v12000> cached{nullptr};
+    PFN_cuTensorMapEncodeTiled_v12000 fn = cached.load(std::memory_order_acquire);
+    if (!fn) {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess) {
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+            cached.store(fn, std::memory_order_release);
+        }
+    }
+    return fn;
+}
 
 // ---------------------------------------------------------------------------
 // device helpers

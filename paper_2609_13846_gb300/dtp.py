@@ -172,6 +172,54 @@ def affinity_workspace(T: int, d: int, H_kv: int, N: int, dtype: int, device) ->
     return torch.empty(affinity_workspace_size(T, d, H_kv, N, dtype), dtype=torch.uint8, device=device)
 
 
+def _cuda_contig(device, **tensors):
+    """Every tensor contiguous and on ``device`` (a CUDA device), else ValueError."""
+    for name, t in tensors.items():
+        if not t.is_cuda or not t.is_contiguous() or t.device != device:
+            raise ValueError(f"{name} must be a contiguous CUDA tensor on the inputs' device")
+
+
+def _add_shapes(C, W_gate, W_up):
+    """C [H,T,d], W_gate/W_up [N,d], all bf16 CUDA tensors on one device; returns (H, T, d, N)."""
+    if not C.is_cuda:
+        raise ValueError("C must be a contiguous CUDA tensor")
+    _cuda_contig(C.device, C=C, W_gate=W_gate, W_up=W_up)
+    if not (C.dtype == W_gate.dtype == W_up.dtype == torch.bfloat16):
+        raise TypeError("C, W_gate and W_up must be bf16")
+    if C.dim() != 3 or W_gate.dim() != 2:
+        raise ValueError("shapes must be C [H,T,d], W_gate [N,d], W_up [N,d]")
+    H, T, d = C.shape
+    N = W_gate.shape[0]
+    if W_gate.shape != (N, d) or W_up.shape != (N, d):
+        raise ValueError("shapes must be C [H,T,d], W_gate [N,d], W_up [N,d]")
+    return H, T, d, N
+
+
+def _check_f32_out(name, t, shape, device):
+    if t.shape != shape or t.dtype != torch.float32 or not t.is_contiguous() or t.device != device:
+        raise ValueError(f"{name} must be a contiguous fp32 {list(shape)} tensor on X's device")
+
+
+def _affinity_shapes(X, C, W_gate, W_up):
+    """Check the affinity inputs (contiguous CUDA tensors of one dtype on one device, X [T,d],
+    C [H,T,d], W_gate/W_up [N,d]) and return (T, d, H, N)."""
+    for name, t in (("X", X), ("C", C), ("W_gate", W_gate), ("W_up", W_up)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+        if t.device != X.device:
+            raise ValueError(f"{name} must be on X's device")
+    if not (X.dtype == C.dtype == W_gate.dtype == W_up.dtype):
+        raise TypeError("X, C, W_gate and W_up must share one dtype")
+    if X.dim() != 2 or C.dim() != 3:
+        raise ValueError("shapes must be X [T,d], C [H,T,d], W_gate [N,d], W_up [N,d]")
+    T, d = X.shape
+    H = C.shape[0]
+    N = W_gate.shape[0]
+    if C.shape != (H, T, d) or W_gate.shape != (N, d) or W_up.shape != (N, d):
+        raise ValueError("shapes must be X [T,d], C [H,T,d], W_gate [N,d], W_up [N,d]")
+    return T, d, H, N
+
+
 def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.Tensor,
                         A: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
                         stream=None, max_ctas: int = 0, defer_reduce: bool = False) -> torch.Tensor:
@@ -183,16 +231,7 @@ def affinity_accumulate(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Tensor, 
     to an even count, at least 2, when the kernel runs as CTA pairs); with defer_reduce only the
     main kernel runs and affinity_reduce(workspace, ...) finishes A later.
     """
-    for name, t in (("X", X), ("C", C), ("W_gate", W_gate), ("W_up", W_up)):
-        if not t.is_cuda or not t.is_contiguous():
-            raise ValueError(f"{name} must be a contiguous CUDA tensor")
-    if not (X.dtype == C.dtype == W_gate.dtype == W_up.dtype):
-        raise TypeError("X, C, W_gate and W_up must share one dtype")
-    T, d = X.shape
-    H = C.shape[0]
-    N = W_gate.shape[0]
-    if C.shape != (H, T, d) or W_gate.shape != (N, d) or W_up.shape != (N, d):
-        raise ValueError("shapes must be X [T,d], C [H,T,d], W_gate [N,d], W_up [N,d]")
+    T, d, H, N = _affinity_shapes(X, C, W_gate, W_up)
     code = _dtype_code(X)
     if A is None:
         A = torch.zeros((H, N), dtype=torch.float32, device=X.device)
@@ -247,16 +286,15 @@ def affinity_accumulate_down(X: torch.Tensor, C: torch.Tensor, W_gate: torch.Ten
     (silu(g_k) u_k)^2 / rms_next[t]^2 with rms_next [T] fp32 the rms of the
     residual entering the next layer's pre-norm.  Returns (A, act2).
     """
-    T, d = X.shape
-    H = C.shape[0]
-    N = W_gate.shape[0]
+    T, d, H, N = _affinity_shapes(X, C, W_gate, W_up)
     code = _dtype_code(X)
     if A is None:
         A = torch.zeros((H, N), dtype=torch.float32, device=X.device)
     if act2 is None:
         act2 = torch.zeros(N, dtype=torch.float32, device=X.device)
-    if rms_next.shape != (T,) or rms_next.dtype != torch.float32:
-        raise ValueError("rms_next must be fp32 [T]")
+    _check_f32_out("A", A, (H, N), X.device)
+    _check_f32_out("act2", act2, (N,), X.device)
+    _check_f32_out("rms_next", rms_next, (T,), X.device)
     if workspace is None:
         workspace = affinity_workspace(T, d, H, N, code, X.device)
     st = lib().dtp_affinity_accumulate_ex(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), _ptr(rms_next), T, d, H, N,
@@ -284,26 +322,18 @@ def affinity_accumulate_grouped(X: torch.Tensor, C_q: torch.Tensor, W_gate: torc
     added to act2 [N] as in affinity_accumulate_down.  Returns A, or (A, act2)
     when rms_next is given.
     """
-    for name, t in (("X", X), ("C_q", C_q), ("W_gate", W_gate), ("W_up", W_up)):
-        if not t.is_cuda or not t.is_contiguous():
-            raise ValueError(f"{name} must be a contiguous CUDA tensor")
-    if not (X.dtype == C_q.dtype == W_gate.dtype == W_up.dtype):
-        raise TypeError("X, C_q, W_gate and W_up must share one dtype")
-    T, d = X.shape
-    Hq = C_q.shape[0]
-    N = W_gate.shape[0]
-    if C_q.shape != (Hq, T, d) or W_gate.shape != (N, d) or W_up.shape != (N, d):
-        raise ValueError("shapes must be X [T,d], C_q [H_q,T,d], W_gate [N,d], W_up [N,d]")
+    T, d, Hq, N = _affinity_shapes(X, C_q, W_gate, W_up)
     if q_per_group < 1 or Hq % q_per_group:
         raise ValueError("q_per_group must divide H_q")
     code = _dtype_code(X)
     if A is None:
         A = torch.zeros((Hq // q_per_group, N), dtype=torch.float32, device=X.device)
+    _check_f32_out("A", A, (Hq // q_per_group, N), X.device)
     if rms_next is not None:
-        if rms_next.shape != (T,) or rms_next.dtype != torch.float32:
-            raise ValueError("rms_next must be fp32 [T]")
+        _check_f32_out("rms_next", rms_next, (T,), X.device)
         if act2 is None:
             act2 = torch.zeros(N, dtype=torch.float32, device=X.device)
+        _check_f32_out("act2", act2, (N,), X.device)
     if workspace is None:
         workspace = _keep(torch.empty(affinity_grouped_workspace_size(T, d, Hq, q_per_group, N, code),
                                       dtype=torch.uint8, device=X.device), stream)
@@ -319,12 +349,12 @@ def affinity_add_accumulate_grouped(C_q: torch.Tensor, W_gate: torch.Tensor, W_u
                                     A_add: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
                                     stream=None) -> torch.Tensor:
     """ADD score per query head, summed over each KV group's query heads (Sec. 3); bf16 inputs."""
-    Hq, T, d = C_q.shape
-    N = W_gate.shape[0]
+    Hq, T, d, N = _add_shapes(C_q, W_gate, W_up)
     if q_per_group < 1 or Hq % q_per_group:
         raise ValueError("q_per_group must divide H_q")
     if A_add is None:
         A_add = torch.zeros((Hq // q_per_group, N), dtype=torch.float32, device=C_q.device)
+    _check_f32_out("A_add", A_add, (Hq // q_per_group, N), C_q.device)
     if workspace is None:
         n = _sz(0)
         _check("dtp_affinity_add_grouped_workspace_size",
@@ -340,10 +370,10 @@ def affinity_add_accumulate(C: torch.Tensor, W_gate: torch.Tensor, W_up: torch.T
                             A_add: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
                             stream=None) -> torch.Tensor:
     """ADD score before the mean (Sec. 3): A_add[h,k] += sum_t (p_h.w^g_k)^2 + (p_h.w^u_k)^2; bf16 inputs."""
-    H, T, d = C.shape
-    N = W_gate.shape[0]
+    H, T, d, N = _add_shapes(C, W_gate, W_up)
     if A_add is None:
         A_add = torch.zeros((H, N), dtype=torch.float32, device=C.device)
+    _check_f32_out("A_add", A_add, (H, N), C.device)
     if workspace is None:
         n = _sz(0)
         _check("dtp_affinity_add_workspace_size", lib().dtp_affinity_add_workspace_size(T, d, H, N, ctypes.byref(n)))
@@ -361,8 +391,17 @@ def down_weight_sqnorm(Wqkv_next: torch.Tensor, gamma_next: torch.Tensor, W_down
     Wqkv_next [H_kv, R, d]: the next layer's q/k/v rows of each KV group;
     gamma_next [d]: its pre-norm gain; W_down [d, N].  All bf16.
     """
+    if not W_down.is_cuda:
+        raise ValueError("W_down must be a contiguous CUDA tensor")
+    _cuda_contig(W_down.device, Wqkv_next=Wqkv_next, gamma_next=gamma_next, W_down=W_down)
+    if not (Wqkv_next.dtype == gamma_next.dtype == W_down.dtype):
+        raise TypeError("Wqkv_next, gamma_next and W_down must share one dtype")
+    if Wqkv_next.dim() != 3 or W_down.dim() != 2:
+        raise ValueError("shapes must be Wqkv_next [H_kv,R,d], gamma_next [d], W_down [d,N]")
     H, R, d = Wqkv_next.shape
     N = W_down.shape[1]
+    if gamma_next.shape != (d,) or W_down.shape != (d, N):
+        raise ValueError("shapes must be Wqkv_next [H_kv,R,d], gamma_next [d], W_down [d,N]")
     bn = torch.empty((H, N), dtype=torch.float32, device=W_down.device)
     if workspace is None:
         n = _sz(0)
@@ -377,7 +416,11 @@ def down_weight_sqnorm(Wqkv_next: torch.Tensor, gamma_next: torch.Tensor, W_down
 
 def down_finalize(act2: torch.Tensor, bn: torch.Tensor, T_total: int, stream=None) -> torch.Tensor:
     """S_down[g,k] = act2[k] / T_total * bn[g,k] (Sec. 3), stored [H_kv, N]."""
+    if not bn.is_cuda or bn.dim() != 2:
+        raise ValueError("bn must be a CUDA fp32 [H_kv, N] tensor")
     H, N = bn.shape
+    _check_f32_out("bn", bn, (H, N), bn.device)
+    _check_f32_out("act2", act2, (N,), bn.device)
     S = torch.empty((H, N), dtype=torch.float32, device=bn.device)
     _check("dtp_down_finalize", lib().dtp_down_finalize(_ptr(act2), _ptr(bn), H, N, int(T_total), _ptr(S),
                                                         _stream(stream)))
@@ -393,9 +436,10 @@ def affinity_accumulate_noalloc(X: torch.Tensor, C: torch.Tensor, W_gate: torch.
     that overlap on the GPU share the scratch and race.  A device-side failure
     is reported by ``affinity_noalloc_status``, not by this call.
     """
-    T, d = X.shape
-    H = C.shape[0]
-    N = W_gate.shape[0]
+    T, d, H, N = _affinity_shapes(X, C, W_gate, W_up)
+    if X.dtype != torch.bfloat16:
+        raise TypeError("the allocation-free path takes bf16 inputs")
+    _check_f32_out("A", A, (H, N), X.device)
     st = lib().dtp_affinity_accumulate_noalloc(_ptr(X), _ptr(C), _ptr(W_gate), _ptr(W_up), T, d, H, N, _ptr(A),
                                                _stream(stream))
     _check("dtp_affinity_accumulate_noalloc", st)

@@ -16,6 +16,12 @@ def test_affinity_rejects_host_tensors():
         dtp.affinity_accumulate(_bf16(16, 64), _bf16(2, 16, 64), _bf16(128, 64), _bf16(128, 64))
     with pytest.raises(ValueError, match="CUDA"):
         dtp.affinity_accumulate_grouped(_bf16(16, 64), _bf16(4, 16, 64), _bf16(128, 64), _bf16(128, 64), 2)
+    with pytest.raises(ValueError, match="CUDA"):
+        dtp.affinity_accumulate_down(_bf16(16, 64), _bf16(2, 16, 64), _bf16(128, 64), _bf16(128, 64),
+                                     torch.ones(16))
+    with pytest.raises(ValueError, match="CUDA"):
+        dtp.affinity_accumulate_noalloc(_bf16(16, 64), _bf16(2, 16, 64), _bf16(128, 64), _bf16(128, 64),
+                                        torch.zeros(2, 128))
 
 
 def test_head_writes_rejects_bad_inputs():
@@ -61,3 +67,14 @@ def test_affinity_opts_struct_layout():
     assert o.max_ctas == 151 and all(x == 0 for x in o.reserved)
     import ctypes
     assert ctypes.sizeof(dtp.AffinityOpts) == 32          # eight ints, as dtp_affinity_opts in dtp.h
+
+
+def test_add_and_down_edge_reject_host_tensors():
+    with pytest.raises(ValueError, match="CUDA"):
+        dtp.affinity_add_accumulate(_bf16(2, 16, 64), _bf16(128, 64), _bf16(128, 64))
+    with pytest.raises(ValueError, match="CUDA"):
+        dtp.affinity_add_accumulate_grouped(_bf16(4, 16, 64), _bf16(128, 64), _bf16(128, 64), 2)
+    with pytest.raises(ValueError, match="CUDA"):
+        dtp.down_weight_sqnorm(_bf16(2, 24, 64), _bf16(64), _bf16(64, 128))
+    with pytest.raises(ValueError, match="CUDA"):
+        dtp.down_finalize(torch.zeros(128), torch.zeros(2, 128), 16)

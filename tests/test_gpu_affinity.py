@@ -294,3 +294,39 @@ def test_top_group_share_matches_oracle():
     L = synth.make_workload_layer(w, T=2048, device=DEV)
     Aw = dtp.affinity_accumulate(L["X"], L["C"], L["W_gate"], L["W_up"])
     assert float(dtp.top_group_share(Aw)) == pytest.approx(oracle.top_group_share(Aw.cpu().numpy()), rel=1e-12)
+
+
+def test_binding_rejects_mismatched_shapes_before_any_launch():
+    """A C with fewer tokens than X, or weights of another width, would let the kernels read past a
+    buffer: the affinity, ADD and down-edge entry points of the binding refuse them on the host."""
+    X = torch.zeros((64, 32), dtype=torch.bfloat16, device=DEV)
+    C_short = torch.zeros((2, 48, 32), dtype=torch.bfloat16, device=DEV)
+    W = torch.zeros((16, 32), dtype=torch.bfloat16, device=DEV)
+    W_wide = torch.zeros((16, 40), dtype=torch.bfloat16, device=DEV)
+    rms = torch.ones(64, device=DEV)
+    A = torch.zeros((2, 16), device=DEV)
+    for C, Wg in ((C_short, W), (torch.zeros((2, 64, 32), dtype=torch.bfloat16, device=DEV), W_wide)):
+        with pytest.raises(ValueError):
+            dtp.affinity_accumulate(X, C, Wg, W)
+        with pytest.raises(ValueError):
+            dtp.affinity_accumulate_down(X, C, Wg, W, rms)
+        with pytest.raises(ValueError):
+            dtp.affinity_accumulate_grouped(X, C, Wg, W, 2)
+        with pytest.raises(ValueError):
+            dtp.affinity_accumulate_noalloc(X, C, Wg, W, A)
+    with pytest.raises(TypeError):
+        dtp.affinity_accumulate_noalloc(X.float(), torch.zeros((2, 64, 32), device=DEV), W.float(), W.float(), A)
+    C = torch.zeros((2, 64, 32), dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(ValueError):
+        dtp.affinity_add_accumulate(C, W_wide, W)
+    with pytest.raises(ValueError):
+        dtp.affinity_add_accumulate_grouped(C, W, W_wide, 2)
+    Wqkv = torch.zeros((2, 24, 32), dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(ValueError):
+        dtp.down_weight_sqnorm(Wqkv, torch.ones(40, dtype=torch.bfloat16, device=DEV),
+                               torch.zeros((32, 16), dtype=torch.bfloat16, device=DEV))
+    with pytest.raises(ValueError):
+        dtp.down_weight_sqnorm(Wqkv, torch.ones(32, dtype=torch.bfloat16, device=DEV),
+                               torch.zeros((40, 16), dtype=torch.bfloat16, device=DEV))
+    with pytest.raises(ValueError):
+        dtp.down_finalize(torch.zeros(15, device=DEV), torch.zeros((2, 16), device=DEV), 64)
