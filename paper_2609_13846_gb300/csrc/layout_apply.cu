@@ -13,8 +13,9 @@
 //                        every row  (o columns; element-wise columns whose
 //                        rows are not a multiple of 16 bytes)
 //   gather_cols_staged_kernel  the same for element-wise columns (down
-//                        columns, one per neuron) with 16-byte rows: row tiles
-//                        and the permutation staged in shared memory
+//                        columns, one per neuron) with 16-byte rows of up to
+//                        32 KB: row tiles staged in shared memory, each
+//                        thread's source offsets held in registers
 // The gathers are pure data movement, bound by HBM: every byte is read once
 // and written once with 16-byte accesses where the block width allows it.  A
 // permutation entry outside [0, blocks) is not followed: the element is left
@@ -202,24 +203,26 @@ __global__ void gather_cols_kernel(const uint8_t* __restrict__ src, uint8_t* __r
 }
 
 // Element-wise column gather staged through shared memory (rows of a multiple
-// of 16 bytes whose column blocks are not whole 16-byte words, e.g. one
-// down_proj column per neuron).  Gathering such elements straight from global
-// memory costs one 32-byte L1 sector per element; here each CTA
-//   - copies its layer's permutation into shared memory once,
-//   - streams tiles of R consecutive rows (contiguous in memory) into a ring of
-//     kStagedStages shared buffers with 1-D bulk copies (cp.async.bulk,
-//     completion counted on an mbarrier), one thread issuing them,
-//   - lets each thread own a fixed set of 16-byte output words: it turns the
-//     permutation entries behind a word into shared-memory offsets once per
-//     tile, then walks the tile's rows gathering from shared memory (4-byte
-//     banks) and storing 16-byte words, coalesced across the warp.
-// CTAs take contiguous ranges of the layers x row-tiles list, so a CTA loads
-// a new permutation only when its range crosses into the next layer.  Small
-// CTAs with two stages keep several CTAs per SM and enough bulk copies in
-// flight; tiles of about 16 KB amortise the per-tile barrier.
-constexpr int kStagedThreads = 128;
+// of 16 bytes, at most 32 KB, whose column blocks are not whole 16-byte words,
+// e.g. one down_proj column per neuron).  Gathering such elements straight from
+// global memory costs one 32-byte L1 sector per element; here each CTA
+//   - streams tiles of R consecutive rows (contiguous in memory) into two
+//     shared buffers with 1-D bulk copies (cp.async.bulk, completion counted on
+//     an mbarrier), one thread issuing them,
+//   - lets each thread own fixed 16-byte output words (ow = tid + w * 256,
+//     w < WPT): when its range of tiles enters a layer, the thread reads the
+//     permutation entries behind its words once and keeps their source offsets
+//     in a staged row in registers (16 bits each, two per register),
+//   - then, for every tile, walks the tile's rows gathering its words' elements
+//     from shared memory and storing each word with one 16-byte write,
+//     coalesced across the warp.
+// CTAs take contiguous ranges of the layers x row-tiles list, so a thread reads
+// the permutation again only when its range crosses into the next layer.
+constexpr int kStagedThreads = 256;
 constexpr int kStagedStages = 2;
 constexpr int64_t kStagedTileTarget = 16 * 1024;   // bytes per staged row tile (at least one row)
+constexpr int kStagedMaxWpt = 8;                    // rows of up to 8 * 256 words = 32 KB
+constexpr uint32_t kNoOffset = 0xFFFFu;             // an entry that is not followed (rows < 64 KB)
 
 struct StagedGeom {
     int64_t rows, row_bytes, block_elems, nblocks, perm_stride;
@@ -234,18 +237,17 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
         : "memory");
 }
 
-template <typename E>
+template <typename E, int WPT>
 __global__ void __launch_bounds__(kStagedThreads)
 gather_cols_staged_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst, StagedGeom g,
                           const int32_t* __restrict__ perm, int* status) {
-    constexpr int kPer = static_cast<int>(16 / sizeof(E));
-    constexpr uint32_t kNone = 0xFFFFFFFFu;            // offset of an entry that is not followed
+    constexpr int kPer = static_cast<int>(16 / sizeof(E));   // elements per 16-byte word
+    constexpr int kPairs = kPer / 2;
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bars[kStagedStages];
     __shared__ int abort_flag;
     const uint32_t row_bytes = static_cast<uint32_t>(g.row_bytes);
     const uint32_t stage_bytes = static_cast<uint32_t>(g.tile_rows) * row_bytes;
-    int32_t* perm_s = reinterpret_cast<int32_t*>(smem + kStagedStages * stage_bytes);
     const int tid = threadIdx.x;
     // this CTA's contiguous range of (layer, row tile) items
     const int64_t t_begin = g.total_tiles * blockIdx.x / gridDim.x;
@@ -274,19 +276,38 @@ gather_cols_staged_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__
     if (tid == 0)
         for (int64_t t = t_begin; t < t_end && t < t_begin + kStagedStages; ++t) issue(t);
 
-    int64_t cur_layer = -1;
-    int bad = 0;
     const int words = static_cast<int>(g.row_bytes / 16);
     const uint32_t be = static_cast<uint32_t>(g.block_elems);
     const uint32_t nblocks = static_cast<uint32_t>(g.nblocks);
+    uint32_t off[WPT][kPairs];   // source byte offsets of this thread's words, two per register
+    int64_t cur_layer = -1;
+    int bad = 0;
     int64_t t = t_begin;
     for (; t < t_end; ++t) {
         const int64_t layer = t / g.tiles_per_layer;
-        if (layer != cur_layer) {      // (re)load the layer's permutation; nobody reads perm_s here
+        if (layer != cur_layer) {
             const int32_t* pl = perm + layer * g.perm_stride;
-            for (int64_t b = tid; b < g.nblocks; b += kStagedThreads) perm_s[b] = pl[b];
+#pragma unroll
+            for (int w = 0; w < WPT; ++w) {
+                const int ow = tid + w * kStagedThreads;
+#pragma unroll
+                for (int i = 0; i < kPairs; ++i) {
+                    uint32_t two[2] = {kNoOffset, kNoOffset};
+                    if (ow < words) {
+#pragma unroll
+                        for (int k = 0; k < 2; ++k) {
+                            const uint32_t c = static_cast<uint32_t>(ow) * kPer + 2 * i + k;
+                            const uint32_t b = c / be;
+                            const int32_t pb = __ldg(pl + b);
+                            const bool ok = static_cast<uint32_t>(pb) < nblocks;
+                            bad |= !ok;
+                            if (ok) two[k] = (static_cast<uint32_t>(pb) * be + (c - b * be)) * sizeof(E);
+                        }
+                    }
+                    off[w][i] = two[0] | (two[1] << 16);
+                }
+            }
             cur_layer = layer;
-            __syncthreads();
         }
         const int st = static_cast<int>((t - t_begin) % kStagedStages);
         const uint32_t parity = static_cast<uint32_t>(((t - t_begin) / kStagedStages) & 1);
@@ -298,47 +319,25 @@ gather_cols_staged_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__
         const int nr = tile_rows_of(t);
         const int64_t r0 = (t % g.tiles_per_layer) * g.tile_rows;
         uint8_t* out = dst + (layer * g.rows + r0) * g.row_bytes;
-        for (int ow = tid; ow < words; ow += kStagedThreads) {
-            // byte offsets in a staged row of the kPer source elements behind output word ow
-            uint32_t off[kPer];
-            if (kPer % 4 == 0 && be == 1) {
-                const int4* pv = reinterpret_cast<const int4*>(perm_s + ow * kPer);
 #pragma unroll
-                for (int q = 0; q < kPer / 4; ++q) {
-                    const int4 p4 = pv[q];
-                    const int32_t pe[4] = {p4.x, p4.y, p4.z, p4.w};
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const bool ok = static_cast<uint32_t>(pe[k]) < nblocks;
-                        bad |= !ok;
-                        off[4 * q + k] = ok ? static_cast<uint32_t>(pe[k]) * sizeof(E) : kNone;
-                    }
-                }
-            } else {
-#pragma unroll
-                for (int i = 0; i < kPer; ++i) {
-                    const uint32_t c = static_cast<uint32_t>(ow) * kPer + i;
-                    const uint32_t b = c / be;
-                    const int32_t pb = perm_s[b];
-                    const bool ok = static_cast<uint32_t>(pb) < nblocks;
-                    bad |= !ok;
-                    off[i] = ok ? (static_cast<uint32_t>(pb) * be + (c - b * be)) * sizeof(E) : kNone;
-                }
-            }
+        for (int w = 0; w < WPT; ++w) {
+            const int ow = tid + w * kStagedThreads;
+            if (ow >= words) continue;
             const uint8_t* rowp = tile;
             uint8_t* op = out + static_cast<int64_t>(ow) * 16;
-#pragma unroll 2
             for (int r = 0; r < nr; ++r) {
-                union { uint4 v; E e[kPer]; } w;
+                union { uint4 v; E e[kPer]; } wd;
 #pragma unroll
-                for (int i = 0; i < kPer; ++i)
-                    w.e[i] = off[i] != kNone ? *reinterpret_cast<const E*>(rowp + off[i]) : E(0);
-                *reinterpret_cast<uint4*>(op) = w.v;
+                for (int i = 0; i < kPer; ++i) {
+                    const uint32_t o = (i & 1) ? (off[w][i >> 1] >> 16) : (off[w][i >> 1] & 0xFFFFu);
+                    wd.e[i] = o != kNoOffset ? *reinterpret_cast<const E*>(rowp + o) : E(0);
+                }
+                *reinterpret_cast<uint4*>(op) = wd.v;
                 rowp += row_bytes;
                 op += g.row_bytes;
             }
         }
-        // every thread is done with this stage (and with perm_s before a reload): refill it
+        // every thread is done with this stage: refill it
         __syncthreads();
         if (tid == 0 && t + kStagedStages < t_end) issue(t + kStagedStages);
     }
@@ -427,10 +426,10 @@ static void cols_by_elem_any(const uint8_t* s, uint8_t* d, int layers, int64_t r
         cols_by_elem<uint8_t>(s, d, layers, rows, row_bytes, block_bytes, perm, perm_stride, status, grid, pack, stream);
 }
 
-template <typename E>
+template <typename E, int WPT>
 static int launch_staged_as(const uint8_t* s, uint8_t* d, const StagedGeom& g, size_t smem, const int32_t* perm,
                             int* status, cudaStream_t stream) {
-    auto* fn = gather_cols_staged_kernel<E>;
+    auto* fn = gather_cols_staged_kernel<E, WPT>;
     DTP_CUDA_TRY(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
     int dev = 0, sms = 0, per_sm = 0;
     DTP_CUDA_TRY(cudaGetDevice(&dev));
@@ -444,11 +443,22 @@ static int launch_staged_as(const uint8_t* s, uint8_t* d, const StagedGeom& g, s
     return DTP_OK;
 }
 
-// Returns DTP_ERR_UNSUPPORTED (nothing launched) when a permutation and the
-// stages do not fit in shared memory; the caller then gathers from global memory.
+template <typename E>
+static int launch_staged_words(const uint8_t* s, uint8_t* d, const StagedGeom& g, size_t smem, const int32_t* perm,
+                               int* status, cudaStream_t stream) {
+    const int64_t wpt = (g.row_bytes / 16 + kStagedThreads - 1) / kStagedThreads;
+    if (wpt <= 1) return launch_staged_as<E, 1>(s, d, g, smem, perm, status, stream);
+    if (wpt <= 2) return launch_staged_as<E, 2>(s, d, g, smem, perm, status, stream);
+    if (wpt <= 4) return launch_staged_as<E, 4>(s, d, g, smem, perm, status, stream);
+    return launch_staged_as<E, kStagedMaxWpt>(s, d, g, smem, perm, status, stream);
+}
+
+// Returns DTP_ERR_UNSUPPORTED (nothing launched) when the rows are wider than the staged kernel
+// handles (32 KB); the caller then gathers from global memory.
 static int launch_cols_staged(const uint8_t* s, uint8_t* d, int layers, int64_t rows, int64_t row_bytes,
                               int64_t block_elems, int elem_bytes, const int32_t* perm, int64_t perm_stride,
                               int* status, cudaStream_t stream) {
+    if (row_bytes > static_cast<int64_t>(kStagedMaxWpt) * kStagedThreads * 16) return DTP_ERR_UNSUPPORTED;
     StagedGeom g;
     g.rows = rows;
     g.row_bytes = row_bytes;
@@ -462,14 +472,13 @@ static int launch_cols_staged(const uint8_t* s, uint8_t* d, int layers, int64_t 
     g.tile_rows = static_cast<int>(tr);
     g.tiles_per_layer = static_cast<int>((rows + tr - 1) / tr);
     g.total_tiles = static_cast<int64_t>(layers) * g.tiles_per_layer;
-    const size_t smem = static_cast<size_t>(kStagedStages) * static_cast<size_t>(tr * row_bytes) +
-                        align_up(static_cast<size_t>(g.nblocks) * 4, 16);
-    if (smem > 200 * 1024 || tr * row_bytes > (int64_t(1) << 30) || g.total_tiles < 1) return DTP_ERR_UNSUPPORTED;
+    const size_t smem = static_cast<size_t>(kStagedStages) * static_cast<size_t>(tr * row_bytes);
+    if (g.total_tiles < 1) return DTP_ERR_UNSUPPORTED;
     switch (elem_bytes) {
-        case 1: return launch_staged_as<uint8_t>(s, d, g, smem, perm, status, stream);
-        case 2: return launch_staged_as<uint16_t>(s, d, g, smem, perm, status, stream);
-        case 4: return launch_staged_as<uint32_t>(s, d, g, smem, perm, status, stream);
-        default: return launch_staged_as<uint64_t>(s, d, g, smem, perm, status, stream);
+        case 1: return launch_staged_words<uint8_t>(s, d, g, smem, perm, status, stream);
+        case 2: return launch_staged_words<uint16_t>(s, d, g, smem, perm, status, stream);
+        case 4: return launch_staged_words<uint32_t>(s, d, g, smem, perm, status, stream);
+        default: return launch_staged_words<uint64_t>(s, d, g, smem, perm, status, stream);
     }
 }
 
