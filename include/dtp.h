@@ -553,9 +553,11 @@ int dtp_layout_order(const int32_t* labels, int layers, int n, int D, int balanc
  *     elements of elem_bytes bytes; o_proj (block = query heads per group *
  *     head_dim columns), down_proj (block = 1 column per neuron)
  *   perm  int32, device, layer i's entries at perm + i * perm_layer_stride
- * An entry of perm outside [0, blocks) is not followed: the affected elements
- * are left unwritten and DTP_ERR_ARG is reported through the workspace status
- * word.  Workspace: dtp_head_writes_workspace_size bytes.  Asynchronous.
+ * An entry of perm outside [0, blocks) is not followed (nothing is read
+ * through it): the affected elements of dst are left unwritten or, where dst
+ * is written in 16-byte words that they share with valid elements, set to
+ * zero, and DTP_ERR_ARG is reported through the workspace status word.
+ * Workspace: dtp_head_writes_workspace_size bytes.  Asynchronous.
  */
 int dtp_permute_rows(const void* src, void* dst, int layers, int64_t rows, int64_t row_bytes, int block_rows,
                      const int32_t* perm, int64_t perm_layer_stride, void* workspace, size_t workspace_bytes,

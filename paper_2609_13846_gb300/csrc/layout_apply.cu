@@ -19,7 +19,8 @@
 // The gathers are pure data movement, bound by HBM: every byte is read once
 // and written once with 16-byte accesses where the block width allows it.  A
 // permutation entry outside [0, blocks) is not followed: the element is left
-// unwritten and DTP_ERR_ARG is set in the status word.
+// unwritten (or, where elements are written as 16-byte words, set to zero) and
+// DTP_ERR_ARG is set in the status word.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
