@@ -235,6 +235,32 @@ def oracle_model_search(A_model, gpu_results, iters):
     return out
 
 
+def model_cpu_baseline(w, S_up, S_down, chain_gpu, searches):
+    """The oracle beside a whole-model run, on the host cores: its affinity on a token slice of layer 0
+    (256 tokens, 64 for the Llama-shaped layer), extrapolated to every layer's tokens, and its
+    whole-model coordinate ascent (both edges) on the GPU's matrices, timed and checked layout for
+    layout against the GPU's; the host times also go into each search entry."""
+    import oracle
+    T_slice = 64 if w.d >= 4096 else 256
+    L = synth.make_workload_layer(w, 0, T=T_slice)
+    X, C, Wg, Wu = (L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up"))
+    t0 = time.perf_counter()
+    oracle.affinity_fo(X, C, Wg, Wu)
+    per_tok = (time.perf_counter() - t0) / T_slice
+    Su = S_up.cpu().numpy()
+    Sd = S_down.cpu().numpy() if S_down is not None else None
+    for D, ref in chain_gpu.items():
+        t0 = time.perf_counter()
+        r = oracle.chain_search(Su, Sd, D, w.iters)
+        searches[f"D{D}"]["host_ms"] = 1e3 * (time.perf_counter() - t0)
+        searches[f"D{D}"]["host_matches_gpu"] = bool(
+            r["J_q"] == int(ref["J_q"]) and np.array_equal(r["h"], ref["h"]) and np.array_equal(r["nu"], ref["nu"]))
+    return {"value": 1.0 / per_tok, "unit": "tokens/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "s_per_token": per_tok, "whole_model_affinity_s_extrapolated": per_tok * w.T * w.layers,
+            "sample": f"affinity on {T_slice} tokens of layer 0 (fp64); the whole-model search on the host on "
+                      f"the GPU's matrices (search.D*.host_ms)"}
+
+
 def layout_suite(args, w, S_up, S_down, S_add, stream):
     """The layouts of Table 4 on this model's affinities at one device count: the optimised layout,
     the ablations (anti-optimised, heads only, neurons only, 4/8/12 evenly spaced layers), the ADD-score
@@ -413,6 +439,7 @@ def run_model(args):
     if Lyr == 1:
         S_down = S_up[:0]
     searches = {}
+    chain_gpu = {}
     for D in w.D:
         r = dtp.search_chain(S_up, S_down if Lyr > 1 else None, D, w.iters)
         torch.cuda.synchronize()
@@ -424,6 +451,7 @@ def run_model(args):
         torch.cuda.synchronize()
         searches[f"D{D}"] = {"ms": s0.elapsed_time(s1) / 3, "J": float(r["J"]), "J_random": (2 * Lyr - 1) / D,
                              "iters_done": int(r["iters_done"])}
+        chain_gpu[D] = {k: r[k].cpu().numpy() for k in ("h", "nu", "J_q")}
     share = dtp.top_group_share(S_up).cpu()              # Sec. 5: largest KV group's share per neuron
     suite, (h_opt, nu_opt, D_opt) = layout_suite(args, w, S_up, S_down, S_add if args.add_score else None, stream)
     apply = time_apply(w, h_opt, nu_opt, D_opt, stream)
@@ -446,6 +474,8 @@ def run_model(args):
             "paper_context": "RTX 5090: affinity 49-51 s (incl. calibration forward), optimisation 38-47 s",
             "clocks": clk.summary(),
             "clocks_note": "sampled over the per-layer scoring loop (input generation included)"}
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = model_cpu_baseline(w, S_up, S_down if Lyr > 1 else None, chain_gpu, searches)
     print(json.dumps(line), flush=True)
 
 
