@@ -194,3 +194,25 @@ def test_down_column_gather_at_model_size(layers, rows, cols):
     ref = torch.gather(src, 2, perm.long().unsqueeze(1).expand(layers, rows, cols))
     assert torch.equal(got, ref)
 
+
+
+@pytest.mark.parametrize("dtype,rows,cols", [(torch.bfloat16, 40, 3072), (torch.float32, 9, 100)])
+def test_column_gather_with_padded_permutation_rows(dtype, rows, cols):
+    """Through the C ABI with perm_layer_stride larger than the permutation (layers' entries padded
+    apart, as a C caller may lay them out): each layer uses its own entries only."""
+    layers, pad = 3, 5
+    g = torch.Generator().manual_seed(cols)
+    src = torch.randint(0, 250, (layers, rows, cols), generator=g).to(dtype).to(DEV)
+    perms = [torch.randperm(cols, generator=g) for _ in range(layers)]
+    padded = torch.full((layers, cols + pad), -7, dtype=torch.int32)   # padding would be out of range
+    for i, p in enumerate(perms):
+        padded[i, :cols] = p.to(torch.int32)
+    padded = padded.to(DEV)
+    dst = torch.empty_like(src)
+    ws = torch.zeros(256, dtype=torch.uint8, device=DEV)
+    st = dtp.lib().dtp_permute_cols(dtp._ptr(src), dtp._ptr(dst), layers, rows, cols, src.element_size(), 1,
+                                    dtp._ptr(padded), cols + pad, dtp._ptr(ws), ws.numel(), dtp._stream(None))
+    assert st == dtp.DTP_OK
+    assert dtp.workspace_status(ws) == dtp.DTP_OK
+    for i, p in enumerate(perms):
+        assert torch.equal(dst[i].cpu(), src[i].cpu()[:, p])
