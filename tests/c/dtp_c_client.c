@@ -2,10 +2,14 @@
  * A plain C client of libdtp: reads X [T,d], C [H,T,d], W_gate, W_up [N,d] (fp32, raw, in that
  * order) from argv[1], runs the first-order affinity pass and the one-layer layout search
  * through the C ABI only, and writes A [H,N] (fp32), h [H], nu [N] (int32) and score_q (int64)
- * to argv[2].  Sizes come from argv[3..7]: T d H N D.
+ * to argv[2].  Sizes come from argv[3..7]: T d H N D.  It then rounds the inputs to bf16 and runs
+ * the bf16 pass twice, with a workspace and through the allocation-free entry point, and prints
+ * whether the two results are equal bit for bit and the allocation-free call's device status.
  */
+#include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
+#include <string.h>
 
 #include <cuda_runtime.h>
 
@@ -19,6 +23,14 @@
             return 1;                                                           \
         }                                                                       \
     } while (0)
+
+/* fp32 -> bf16, round to nearest even (finite inputs) */
+static uint16_t to_bf16(float f) {
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
 
 static int read_all(const char* path, float* dst, size_t n) {
     FILE* f = fopen(path, "rb");
@@ -87,5 +99,35 @@ int main(int argc, char** argv) {
     fwrite(&sq, sizeof(int64_t), 1, f);
     fclose(f);
     printf("ok %lld\n", (long long)sq);
+
+    /* bf16: the workspace entry point and the allocation-free one on the same inputs */
+    const size_t ntot = nx + nc + 2 * nw;
+    uint16_t* hb = (uint16_t*)malloc(sizeof(uint16_t) * ntot);
+    if (!hb) return 3;
+    for (size_t i = 0; i < ntot; ++i) hb[i] = to_bf16(host[i]);
+    uint16_t* xb;
+    float *a_ws, *a_na;
+    void* ws_bf = NULL;
+    size_t b_bf = 0;
+    CHECK(dtp_affinity_workspace_size(T, d, H, N, DTP_BF16, &b_bf));
+    CHECK(cudaMalloc((void**)&xb, sizeof(uint16_t) * ntot));
+    CHECK(cudaMalloc((void**)&a_ws, sizeof(float) * (size_t)H * N));
+    CHECK(cudaMalloc((void**)&a_na, sizeof(float) * (size_t)H * N));
+    CHECK(cudaMalloc(&ws_bf, b_bf));
+    CHECK(cudaMemcpy(xb, hb, sizeof(uint16_t) * ntot, cudaMemcpyHostToDevice));
+    CHECK(cudaMemset(a_ws, 0, sizeof(float) * (size_t)H * N));
+    CHECK(cudaMemset(a_na, 0, sizeof(float) * (size_t)H * N));
+    CHECK(dtp_affinity_accumulate(xb, xb + nx, xb + nx + nc, xb + nx + nc + nw, T, d, H, N, DTP_BF16, a_ws, ws_bf,
+                                  b_bf, NULL));
+    CHECK(dtp_affinity_accumulate_noalloc(xb, xb + nx, xb + nx + nc, xb + nx + nc + nw, T, d, H, N, a_na, NULL));
+    const int na_status = dtp_affinity_noalloc_status(NULL);
+    CHECK(cudaDeviceSynchronize());
+    CHECK(dtp_workspace_status(ws_bf, b_bf, NULL));
+    float* A1 = (float*)malloc(sizeof(float) * (size_t)H * N);
+    float* A2 = (float*)malloc(sizeof(float) * (size_t)H * N);
+    if (!A1 || !A2) return 3;
+    CHECK(cudaMemcpy(A1, a_ws, sizeof(float) * (size_t)H * N, cudaMemcpyDeviceToHost));
+    CHECK(cudaMemcpy(A2, a_na, sizeof(float) * (size_t)H * N, cudaMemcpyDeviceToHost));
+    printf("noalloc_equal %d status %d\n", memcmp(A1, A2, sizeof(float) * (size_t)H * N) == 0, na_status);
     return 0;
 }

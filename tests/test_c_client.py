@@ -1,5 +1,6 @@
 """The C ABI used from plain C: the header compiles as strict C99, and (on a GPU) a C client that
-allocates with cudaMalloc and calls only libdtp reproduces the Python binding bit for bit."""
+allocates with cudaMalloc and calls only libdtp reproduces the Python binding bit for bit, and its
+bf16 pass through the allocation-free entry point equals the workspace entry point's."""
 import os
 import shutil
 import subprocess
@@ -67,3 +68,6 @@ def test_c_client_matches_the_binding():
     assert sq_c == int(lay["score_q"])
     ref = oracle.affinity_fo(*(L[k].double().numpy() for k in ("X", "C", "W_gate", "W_up")))
     assert np.linalg.norm(A_c - ref) / np.linalg.norm(ref) <= 1e-5
+    # bf16 through plain C: the allocation-free entry point equals the workspace one bit for bit and
+    # its status reader reports DTP_OK
+    assert "noalloc_equal 1 status 0" in run.stdout, run.stdout
