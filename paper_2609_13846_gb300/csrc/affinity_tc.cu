@@ -442,7 +442,7 @@ affinity_fo_tc_kernel(const __grid_constant__ CUtensorMap tm_wg, const __grid_co
             __syncwarp();
             if (lane == 0) {
                 if constexpr (kPair)
-                    mbar_arrive_cluster(mapa_shared(smem_u32(&acc_empty[buf]), 0));
+                    mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&acc_empty[buf]), 0));
                 else
                     mbar_arrive(smem_u32(&acc_empty[buf]));
             }

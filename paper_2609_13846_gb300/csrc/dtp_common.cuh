@@ -265,6 +265,15 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
+// Relaxed arrive on an mbarrier given by its shared::cluster address.  Used where the arriving
+// thread hands a TMEM accumulator back to the MMA thread after tcgen05.wait::ld: its TMEM reads
+// have completed before the arrive is issued, so no release ordering is needed for the MMAs
+// that overwrite the buffer, and the arrive does not wait for this thread's other memory
+// operations (shared stores of partial sums, bulk stores) to become visible cluster-wide.
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
