@@ -280,9 +280,11 @@ head_writes_tc_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_con
                 }
                 sbuf ^= 1u;
             }
+            // its TMEM loads have completed (tcgen05.wait::ld): hand the buffer back without release
+            // ordering, which would also wait for the warp's staging stores
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+            if (lane == 0) mbar_arrive_relaxed(smem_u32(&acc_empty[buf]));
         }
         if (lane == 0) bulk_wait_all();
         __syncwarp();
