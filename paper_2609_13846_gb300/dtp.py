@@ -197,7 +197,7 @@ def _add_shapes(C, W_gate, W_up):
 
 def _check_f32_out(name, t, shape, device):
     if t.shape != shape or t.dtype != torch.float32 or not t.is_contiguous() or t.device != device:
-        raise ValueError(f"{name} must be a contiguous fp32 {list(shape)} tensor on X's device")
+        raise ValueError(f"{name} must be a contiguous fp32 {list(shape)} tensor on the inputs' device")
 
 
 def _affinity_shapes(X, C, W_gate, W_up):
