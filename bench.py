@@ -19,6 +19,7 @@ Rank 0 prints one JSON line.
 from __future__ import annotations
 
 import argparse
+import datetime
 import json
 import os
 import statistics
@@ -75,9 +76,12 @@ def traffic_from_profile():
 
 
 class Clocks:
-    """Samples nvidia-smi clocks and throttle reasons during the timed region."""
+    """Samples nvidia-smi clocks and throttle reasons during the timed region.
 
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    mark_start() / mark_end() bracket the timed work; the summary uses the samples taken between
+    the two marks (by nvidia-smi's own timestamps) when there are any, else every sample."""
+
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -85,6 +89,7 @@ class Clocks:
         self.gpu = gpu_index
         self.proc = None
         self.path = None
+        self.t0 = self.t1 = None
 
     def __enter__(self):
         # samples go to a git-ignored folder of the repository
@@ -94,11 +99,17 @@ class Clocks:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+                 "-lms", "50"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except (FileNotFoundError, OSError):
             self.proc = None
         time.sleep(0.25)
         return self
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
 
     def __exit__(self, *exc):
         if self.proc is not None:
@@ -111,24 +122,31 @@ class Clocks:
     def summary(self):
         if self.proc is None or not self.path:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm, smax, reasons = [], None, set()
+        rows, smax = [], None
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in open(self.path):
             parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 9:
+            if len(parts) < 10:
                 continue
             try:
-                sm.append(float(parts[1]))
-                smax = float(parts[2])
+                sm = float(parts[2])
+                smax = float(parts[3])
             except ValueError:
                 continue
-            for name, val in zip(names, parts[5:9]):
-                if val.lower().startswith("active"):
-                    reasons.add(name)
+            try:
+                ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+            except ValueError:
+                ts = None       # an unexpected timestamp format: the sample still counts, outside the window
+            rows.append((ts, sm, {n for n, v in zip(names, parts[6:10]) if v.lower().startswith("active")}))
         os.unlink(self.path)
-        busy = [s for s in sm if smax and s > 0.3 * smax] or sm
+        inside = [r for r in rows
+                  if r[0] is not None and self.t0 is not None and self.t1 is not None and self.t0 <= r[0] <= self.t1]
+        use = inside or rows
+        sm = [r[1] for r in use]
+        reasons = set().union(*[r[2] for r in use]) if use else set()
+        busy = [x for x in sm if smax and x > 0.3 * smax] or sm
         return {"sm_mhz": statistics.median(busy) if busy else None, "sm_max_mhz": smax,
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "reasons": sorted(reasons), "samples": len(rows), "samples_in_timed_region": len(inside)}
 
 
 def dist_env():
@@ -482,7 +500,7 @@ def run_model(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work for cpu_baseline")
@@ -578,12 +596,14 @@ def main():
     with Clocks(local) as clk:
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
+        clk.mark_start()
         t0.record(stream)
         for _ in range(args.steps):
             res = step(record=True)
         stream.wait_stream(side)                 # the last step's search is inside the timed region
         t1.record(stream)
         torch.cuda.synchronize()
+        clk.mark_end()
     barrier()
     elapsed_ms = shard.max_over_ranks(t0.elapsed_time(t1), device=dev)
     aff_ms = [a.elapsed_time(b) for a, b in aff_ev]
@@ -602,12 +622,14 @@ def main():
         torch.cuda.synchronize()
         with Clocks(local) as clk_s:
             u0, u1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            clk_s.mark_start()
             u0.record(stream)
             for k in range(n_sus):
                 step(record=k >= n_sus // 2)
             stream.wait_stream(side)
             u1.record(stream)
             torch.cuda.synchronize()
+            clk_s.mark_end()
         barrier()
         sus_ms = shard.max_over_ranks(u0.elapsed_time(u1), device=dev)
         sus_aff = float(np.mean([a.elapsed_time(b) for a, b in aff_ev]))
