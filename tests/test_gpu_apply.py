@@ -216,3 +216,25 @@ def test_column_gather_with_padded_permutation_rows(dtype, rows, cols):
     assert dtp.workspace_status(ws) == dtp.DTP_OK
     for i, p in enumerate(perms):
         assert torch.equal(dst[i].cpu(), src[i].cpu()[:, p])
+
+
+def test_row_gather_with_padded_permutation_rows():
+    """dtp_permute_rows through the C ABI with perm_layer_stride larger than the permutation."""
+    layers, rows, cols, block, pad = 3, 48, 64, 2, 3
+    g = torch.Generator().manual_seed(7)
+    src = torch.randint(0, 250, (layers, rows, cols), generator=g).to(torch.bfloat16).to(DEV)
+    nb = rows // block
+    perms = [torch.randperm(nb, generator=g) for _ in range(layers)]
+    padded = torch.full((layers, nb + pad), -3, dtype=torch.int32)
+    for i, p in enumerate(perms):
+        padded[i, :nb] = p.to(torch.int32)
+    padded = padded.to(DEV)
+    dst = torch.empty_like(src)
+    ws = torch.zeros(256, dtype=torch.uint8, device=DEV)
+    st = dtp.lib().dtp_permute_rows(dtp._ptr(src), dtp._ptr(dst), layers, rows, cols * src.element_size(), block,
+                                    dtp._ptr(padded), nb + pad, dtp._ptr(ws), ws.numel(), dtp._stream(None))
+    assert st == dtp.DTP_OK
+    assert dtp.workspace_status(ws) == dtp.DTP_OK
+    for i, p in enumerate(perms):
+        idx = torch.cat([torch.arange(b * block, (b + 1) * block) for b in p.tolist()])
+        assert torch.equal(dst[i].cpu(), src[i].cpu()[idx])
