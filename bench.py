@@ -393,6 +393,7 @@ def run_model(args):
     if args.producer and q not in (1, w.q_per_group):
         raise SystemExit("--producer takes --qheads 1 (KV-group rows) or the model's query heads per group")
     with Clocks(local) as clk:
+        clk.mark_start()
         for li, i in enumerate(mine):
             L = synth.make_workload_layer(w, i, device=dev) if q == 1 else \
                 synth.make_layer(d, G * q, N, T, w.layer_seed(i), dtype=w.dtype, outliers=w.outliers, device=dev)
@@ -440,6 +441,7 @@ def run_model(args):
             if args.add_score:
                 t_add += e2.elapsed_time(e3)
             del L, Dn
+        clk.mark_end()
     if dtp.workspace_status(ws) != dtp.DTP_OK:
         raise RuntimeError("affinity kernel reported a device-side error")
     torch.cuda.synchronize()
