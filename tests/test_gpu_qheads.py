@@ -105,17 +105,22 @@ def test_grouped_add_one_head_per_group_is_plain():
 
 
 def test_grouped_sampled_neurons_at_qwen_size():
-    """The Qwen3-0.6B layer with its 16 query heads (2 per KV group) at 16384 tokens; 48
-    sampled neurons checked against the oracle."""
+    """The Qwen3-0.6B layer with its 16 query heads (2 per KV group) at 16384 tokens; two whole
+    128-neuron tiles (the middle one and the last) and 24 sampled neurons checked against the oracle,
+    by relative Frobenius error and every entry within 2%."""
     w = synth.WORKLOADS["qwen3_0.6b_layer"]
     L = synth.make_layer(w.d, 16, w.N, w.T, seed=w.seed, dtype="bf16", outliers=True, device=DEV)
     A = dtp.affinity_accumulate_grouped(L["X"], L["C"], L["W_gate"], L["W_up"], 2)
     torch.cuda.synchronize()
-    rows = np.random.default_rng(0).choice(w.N, 48, replace=False)
+    mid = (w.N // 128) // 2 * 128
+    rows = np.unique(np.concatenate([np.arange(mid, mid + 128), np.arange(w.N - 128, w.N),
+                                     np.random.default_rng(0).choice(w.N, 24, replace=False)]))
     sub = {k: L[k].cpu() for k in ("X", "C")}
     ref = oracle.affinity_fo_qheads(sub["X"].double().numpy(), sub["C"].double().numpy(),
                                     L["W_gate"][rows].cpu().double().numpy(), L["W_up"][rows].cpu().double().numpy(), 2)
-    assert _rel(A[:, rows].cpu().numpy(), ref) <= BF16_TOL
+    got = A[:, rows].cpu().numpy()
+    assert _rel(got, ref) <= BF16_TOL
+    assert np.all(np.abs(got - ref) <= 2e-2 * np.abs(ref) + 1e-6 * np.abs(ref).max())
 
 
 def test_grouped_rejects_bad_group_sizes():
